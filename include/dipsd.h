@@ -1,0 +1,176 @@
+/*
+ * dipsd.h -- C ABI of the GB300 (sm_103a) batched-verification library for
+ * DiP-SD edge servers (arXiv 2604.20919).
+ *
+ * In every speculative-decoding round each user's device sends L_i draft
+ * tokens to the edge server, which verifies a whole batch of users in one
+ * target-model pass (Sec. II-A, stage 2 "Batch Verification"): it finds each
+ * user's first rejected draft, drops the drafts after it, and emits one more
+ * token after the last accepted position, so every user gets at least one
+ * token per round.  The per-user arguments follow the paper's problem
+ * statement (Sec. II-A, Table 1): draft length l_m (here L_i), prefix length
+ * i_m (here the context length C_i), and batch membership B_n(x)
+ * (Sec. III-C, the users assigned to stage n).
+ *
+ * This library implements the data-parallel part of that step:
+ *   dipsd_verify_attention  causal GQA attention of each user's L_i+1 verify
+ *                           tokens over the user's paged bf16 KV cache;
+ *   dipsd_spec_verify       speculative sampling over the vocabulary;
+ *   dipsd_verify_batch      both, for one pipeline stage's users.
+ *
+ * Conventions shared by every entry point
+ *   - Pointers named d_* are device pointers, h_* host pointers.  The caller
+ *     owns all memory; the library never allocates or frees.
+ *   - Calls are asynchronous on `stream` (a cudaStream_t passed as void*;
+ *     NULL = legacy default stream).  Outputs are valid once the stream has
+ *     reached the end of the call.
+ *   - Every argument is validated on the host before anything is launched;
+ *     on error nothing is written and a status code is returned.
+ *   - Verify token t of user i (t = 0..L_i) is the token at absolute position
+ *     C_i + t: t = 0 is the last token emitted in the previous round, t >= 1
+ *     are the drafts d_{i,1..L_i}.  Tokens are packed user after user in batch
+ *     order: user i's tokens start at row sum_{j<i} (L_j + 1).
+ *   - Workspace: caller-allocated device memory of at least the size the
+ *     matching *_workspace_size call returns for the same per-user arguments
+ *     (on the same device).  Its first 16 bytes hold a device status word:
+ *     kernels OR error bits into it (DIPSD_DEVERR_*) instead of trapping; zero
+ *     it before a call whose status you want to read.  Calls that share a
+ *     workspace must not overlap on the GPU.
+ */
+#ifndef DIPSD_H
+#define DIPSD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define DIPSD_ABI_VERSION 1
+#define DIPSD_PAGE_SIZE 16    /* tokens per KV page */
+#define DIPSD_MAX_USERS 512   /* users per call */
+#define DIPSD_MAX_DRAFT 31    /* L_i <= 31: one warp ballot covers a user */
+
+typedef enum {
+  DIPSD_OK = 0,
+  DIPSD_ERR_INVALID_ARG = 1, /* a size, length or pointer failed validation */
+  DIPSD_ERR_UNSUPPORTED = 2, /* valid but not built (e.g. head_dim not 64/128) */
+  DIPSD_ERR_CUDA = 3,        /* a CUDA runtime call or launch failed */
+  DIPSD_ERR_WORKSPACE = 4    /* workspace NULL, misaligned or too small */
+} dipsd_status;
+
+typedef enum { DIPSD_BF16 = 0, DIPSD_F32 = 1 } dipsd_dtype;
+
+/* Device status bits (workspace word 0). */
+#define DIPSD_DEVERR_WAIT_TIMEOUT 1u /* a bounded mbarrier wait expired */
+#define DIPSD_DEVERR_BAD_TOKEN 2u    /* a draft token outside [0, V): treated as rejected */
+
+/* Human-readable name of a dipsd_status value (static string). */
+const char* dipsd_status_string(int status);
+
+/* DIPSD_ABI_VERSION of the loaded library. */
+int dipsd_abi_version(void);
+
+/* Number of CUDA kernels this library has launched from the calling host
+ * thread since the library was loaded (a diagnostic counter). */
+long long dipsd_launch_count(void);
+
+/* ------------------------------------------------------------------------
+ * Verify attention (the target model's attention over the verify tokens,
+ * Sec. II-A stage 2; its cost is the I*L term of Eq. (Fv)).
+ *
+ * For user i, verify token t and query head h (KV head h / G, G = Hq/Hkv):
+ *   out[t,h] = sum_{j <= C_i + t} softmax_j(softmax_scale * q[t,h] . k_j) v_j
+ * over the user's keys j = 0 .. C_i + L_i.  The K/V rows of the L_i+1 verify
+ * tokens must already be written into the cache pages.
+ *
+ * B             number of users, 1..DIPSD_MAX_USERS
+ * h_L, h_ctx    [B] host: draft length L_i in 0..DIPSD_MAX_DRAFT, context C_i >= 0
+ * d_q           [sum_i (L_i+1)][Hq][D] bf16, row-major, 16-byte aligned
+ * d_k_cache,
+ * d_v_cache     [num_blocks][Hkv][DIPSD_PAGE_SIZE][D] bf16, 16-byte aligned
+ * d_block_table [B][max_blocks] int32: page p of user i (tokens 16p..16p+15)
+ *               is cache block d_block_table[i*max_blocks + p]; entries past
+ *               ceil((C_i+L_i+1)/16) are never read.  A block id outside
+ *               [0, num_blocks) reads zeros (it cannot fault).
+ * Hq, Hkv, D    query heads, KV heads (Hq % Hkv == 0), head_dim in {64, 128}
+ * softmax_scale usually D^-1/2
+ * d_out         [sum_i (L_i+1)][Hq][D] bf16 (may not alias d_q)
+ * Requires C_i + L_i + 1 <= 16 * max_blocks for every user.
+ * ---------------------------------------------------------------------- */
+size_t dipsd_verify_attention_workspace_size(int B, const int* h_L, const int* h_ctx,
+                                             int Hq, int Hkv, int D);
+int dipsd_verify_attention(int B, const int* h_L, const int* h_ctx,
+                           const void* d_q, const void* d_k_cache, const void* d_v_cache,
+                           int num_blocks, const int* d_block_table, int max_blocks,
+                           int Hq, int Hkv, int D, float softmax_scale,
+                           void* d_out, void* d_workspace, size_t workspace_bytes,
+                           void* stream);
+
+/* ------------------------------------------------------------------------
+ * Speculative verification (Sec. II-A stage 2: first-mismatch truncation and
+ * one bonus token; the accept/reject rule is the speculative sampling the
+ * paper cites, whose expected output length is Eq. (u_single)).
+ *
+ * Per user i and draft position t < L_i (draft d = d_{i,t+1}):
+ *   p_t = softmax(target_logits[t]), q_t = softmax(draft_logits[t]),
+ *   accepted iff u_acc(t) * q_t(d) < p_t(d).
+ * a_i = number of leading accepted drafts.  Emitted: d_{i,1..a_i}, then one
+ * token drawn with u_res(a_i) by inverse CDF (smallest k whose cumulative
+ * weight exceeds u * total, ascending token order) from
+ *   max(0, p_a - q_a)  if a_i < L_i (p_a itself if that has no mass),
+ *   p_{L_i}            if a_i == L_i (the bonus position).
+ *
+ * B                  1..DIPSD_MAX_USERS;  h_L [B] host, 0..DIPSD_MAX_DRAFT
+ * V                  vocabulary size >= 1
+ * logit_dtype        DIPSD_BF16 or DIPSD_F32 (both logit arrays)
+ * d_target_logits    [sum_i (L_i+1)][V], user i's rows in position order
+ * d_draft_logits     [sum_i L_i][V]
+ * d_draft_tokens     [sum_i L_i] int32 in [0, V)
+ * d_uniforms         [sum_i (L_i+1)][2] fp32 in (0,1): (u_acc, u_res) per
+ *                    verify position (u_acc of the bonus position is unused)
+ * d_accept_len       [B] int32 out: a_i
+ * d_out_offsets      [B+1] int32 out: exclusive prefix of (a_i + 1)
+ * d_out_tokens       [sum_i (L_i+1)] int32 out (capacity); the first
+ *                    d_out_offsets[B] entries are the packed emitted tokens
+ * d_draft_probs      NULL or [sum_i (L_i+1)][2] fp32 out: (p_t(d), q_t(d)) at
+ *                    every draft position, (0, 0) at bonus positions
+ * Rows must start 16-byte aligned for the fast path (V*elem % 16 == 0).
+ * ---------------------------------------------------------------------- */
+size_t dipsd_spec_verify_workspace_size(int B, const int* h_L, int V);
+int dipsd_spec_verify(int B, const int* h_L, int V, int logit_dtype,
+                      const void* d_target_logits, const void* d_draft_logits,
+                      const int* d_draft_tokens, const float* d_uniforms,
+                      int* d_accept_len, int* d_out_offsets, int* d_out_tokens,
+                      float* d_draft_probs, void* d_workspace, size_t workspace_bytes,
+                      void* stream);
+
+/* ------------------------------------------------------------------------
+ * One pipeline stage: the users of batch n (Sec. III-C, B_n(x)) verified
+ * together -- attention, then speculative verification, on one stream.
+ *
+ * Per-user tables cover all M users being served; h_members[b] (distinct, in
+ * [0, M)) names the b-th user of this batch.  Per-batch tensors (d_q,
+ * d_attn_out, logits, draft tokens, uniforms and the outputs) are packed in
+ * h_members order exactly as for the two calls above.
+ * h_L_all, h_ctx_all  [M] host;  d_block_table_all [M][max_blocks] int32.
+ * ---------------------------------------------------------------------- */
+size_t dipsd_verify_batch_workspace_size(int B, const int* h_members, int M,
+                                         const int* h_L_all, const int* h_ctx_all,
+                                         int Hq, int Hkv, int D, int V);
+int dipsd_verify_batch(int B, const int* h_members, int M,
+                       const int* h_L_all, const int* h_ctx_all,
+                       const void* d_q, const void* d_k_cache, const void* d_v_cache,
+                       int num_blocks, const int* d_block_table_all, int max_blocks,
+                       int Hq, int Hkv, int D, float softmax_scale, void* d_attn_out,
+                       int V, int logit_dtype, const void* d_target_logits,
+                       const void* d_draft_logits, const int* d_draft_tokens,
+                       const float* d_uniforms, int* d_accept_len, int* d_out_offsets,
+                       int* d_out_tokens, float* d_draft_probs,
+                       void* d_workspace, size_t workspace_bytes, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* DIPSD_H */

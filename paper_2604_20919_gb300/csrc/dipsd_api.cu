@@ -1,0 +1,564 @@
+// Host side of the C ABI declared in include/dipsd.h: argument validation,
+// work planning (KV split sizes, cluster sizes, workspace layout), TMA tensor
+// map encoding and kernel launches.  No entry point allocates or synchronises.
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include "dipsd.h"
+#include "attention.cuh"
+#include "spec_verify.cuh"
+
+namespace dipsd {
+namespace {
+
+constexpr size_t kStatusBytes = 256;
+constexpr int kCapSmall = 64;
+constexpr int kCapLarge = kMaxUsers;
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// ------------------------------------------------------------ device facts
+struct DeviceFacts {
+  int sms = 0;
+  int max_smem_optin = 0;
+};
+
+bool device_facts(DeviceFacts& f) {
+  static std::mutex mu;
+  static DeviceFacts cache[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
+  std::lock_guard<std::mutex> lock(mu);
+  if (cache[dev].sms == 0) {
+    if (cudaDeviceGetAttribute(&cache[dev].sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return false;
+    cudaDeviceGetAttribute(&cache[dev].max_smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  }
+  f = cache[dev];
+  return f.sms > 0;
+}
+
+// ------------------------------------------------------ TMA tensor maps
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// Paged cache [num_blocks][Hkv][16][D] bf16 as a 4-D tensor (D innermost);
+// one box = one page of one head, 64 columns wide, 128-byte swizzle.
+bool encode_cache_map(CUtensorMap* map, const void* base, int num_blocks, int Hkv, int D) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return false;
+  cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)kPage, (cuuint64_t)Hkv, (cuuint64_t)num_blocks};
+  cuuint64_t strides[3] = {(cuuint64_t)D * 2, (cuuint64_t)kPage * D * 2, (cuuint64_t)Hkv * kPage * D * 2};
+  cuuint32_t box[4] = {64, (cuuint32_t)kPage, 1, 1};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// --------------------------------------------------------------- launching
+thread_local long long g_launches = 0;
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                   int cluster, bool pdl, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  int n = 0;
+  if (cluster > 0) {
+    attr[n].id = cudaLaunchAttributeClusterDimension;
+    attr[n].val.clusterDim.x = cluster;
+    attr[n].val.clusterDim.y = 1;
+    attr[n].val.clusterDim.z = 1;
+    ++n;
+  }
+  if (pdl) {
+    attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[n].val.programmaticStreamSerializationAllowed = 1;
+    ++n;
+  }
+  cfg.attrs = attr;
+  cfg.numAttrs = n;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+  if (e == cudaSuccess) ++g_launches;
+  return e;
+}
+
+// =================================================================== attention
+struct AttnPlan {
+  int B = 0, Hq = 0, Hkv = 0, G = 0, D = 0;
+  int NW = 4, stages = 3;
+  int n_items = 0, n_merge = 0;
+  long long part_rows = 0;
+  std::vector<AttnUser> u;
+  std::vector<int> item_off, merge_off;
+  std::vector<long long> part_off;
+  size_t smem = 0;
+  size_t ws_bytes = 0;  // attention region only (excludes the status word)
+};
+
+int attn_stages(int D, int NW) { return D == 128 ? (NW == 4 ? 3 : 4) : 4; }
+
+size_t attn_smem(int D, int stages) {
+  return static_cast<size_t>(stages) * 2 * kAttnTile * D * 2 + 2 * stages * sizeof(uint64_t) + 1024;
+}
+
+// Validates the per-user attention arguments.
+int check_attn_users(int B, const int* L, const int* ctx, int Hq, int Hkv, int D) {
+  if (B < 1 || B > kMaxUsers || !L || !ctx) return DIPSD_ERR_INVALID_ARG;
+  if (Hkv < 1 || Hq < Hkv || Hq % Hkv != 0 || Hq > 4096) return DIPSD_ERR_INVALID_ARG;
+  if (D != 64 && D != 128) return D > 0 ? DIPSD_ERR_UNSUPPORTED : DIPSD_ERR_INVALID_ARG;
+  long long sum_t = 0;
+  for (int i = 0; i < B; ++i) {
+    if (L[i] < 0 || L[i] > kMaxDraft || ctx[i] < 0) return DIPSD_ERR_INVALID_ARG;
+    if (static_cast<long long>(ctx[i]) + L[i] + 1 > (1ll << 30)) return DIPSD_ERR_INVALID_ARG;
+    sum_t += L[i] + 1;
+  }
+  if (sum_t * Hq * D > (1ll << 40)) return DIPSD_ERR_INVALID_ARG;
+  return DIPSD_OK;
+}
+
+// Chooses the KV split length (a multiple of the 64-token tile) that
+// minimises a list-scheduling estimate of the makespan over the resident CTA
+// slots: total work / slots + the largest item, with a per-item overhead of
+// two tiles (prologue, pipeline fill, epilogue) and the merge traffic.
+void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int Hq, int Hkv, int D,
+                    int sms, AttnPlan& pl) {
+  pl.B = B; pl.Hq = Hq; pl.Hkv = Hkv; pl.G = Hq / Hkv; pl.D = D;
+  int max_m = 0, max_tiles = 1;
+  for (int i = 0; i < B; ++i) {
+    max_m = std::max(max_m, pl.G * (L[i] + 1));
+    max_tiles = std::max(max_tiles, (ctx[i] + L[i] + 1 + kAttnTile - 1) / kAttnTile);
+  }
+  pl.NW = max_m <= 64 ? 4 : 8;
+  pl.stages = attn_stages(D, pl.NW);
+  pl.smem = attn_smem(D, pl.stages);
+  const int rows_cta = pl.NW * 16;
+  const int per_sm_smem = static_cast<int>((228 * 1024) / (pl.smem + 1024));
+  const int per_sm_regs = 65536 / ((pl.NW + 1) * 32 * 168);
+  const int slots = sms * std::max(1, std::min(per_sm_smem, per_sm_regs));
+
+  int forced = 0;
+  if (const char* e = std::getenv("DIPSD_ATTN_SPLIT_TILES")) forced = std::atoi(e);
+  const int cands[] = {1, 2, 3, 4, 5, 6, 8, 10, 12, 16, 20, 24, 32, 40, 48, 64, 96, 128, 192, 256, 384, 512, 1 << 30};
+  double best = 1e300;
+  int best_c = 1 << 30;
+  for (int c : cands) {
+    if (forced > 0) c = forced;
+    double total = 0, max_item = 0;
+    long long items = 0;
+    for (int i = 0; i < B; ++i) {
+      const int tiles = (ctx[i] + L[i] + 1 + kAttnTile - 1) / kAttnTile;
+      const int cc = std::max(1, std::min(c, tiles));
+      int ns = (tiles + cc - 1) / cc;
+      const int st = (tiles + ns - 1) / ns;
+      ns = (tiles + st - 1) / st;
+      const int rb = (pl.G * (L[i] + 1) + rows_cta - 1) / rows_cta;
+      const double item = st + 2.0 + (ns > 1 ? 0.5 : 0.0);
+      total += item * ns * rb * Hkv;
+      items += static_cast<long long>(ns) * rb * Hkv;
+      max_item = std::max(max_item, item);
+    }
+    if (items > (1ll << 30)) continue;
+    const double cost = total / slots + max_item;
+    if (cost < best - 1e-9) { best = cost; best_c = c; }
+    if (forced > 0) break;
+  }
+
+  pl.u.assign(B, AttnUser{});
+  pl.item_off.assign(B + 1, 0);
+  pl.merge_off.assign(B + 1, 0);
+  pl.part_off.assign(B, -1);
+  long long items = 0, merge = 0, part = 0;
+  for (int i = 0; i < B; ++i) {
+    AttnUser& U = pl.u[i];
+    U.q_off = i == 0 ? 0 : pl.u[i - 1].q_off + pl.u[i - 1].T;
+    U.ctx = ctx[i];
+    U.T = L[i] + 1;
+    U.kv_len = ctx[i] + U.T;
+    U.bt_row = bt_rows ? bt_rows[i] : i;
+    const int tiles = (U.kv_len + kAttnTile - 1) / kAttnTile;
+    const int cc = std::max(1, std::min(best_c, tiles));
+    int ns = (tiles + cc - 1) / cc;
+    const int st = (tiles + ns - 1) / ns;
+    ns = (tiles + st - 1) / st;
+    U.nsplit = ns;
+    U.split_len = st * kAttnTile;
+    U.n_rb = (pl.G * U.T + rows_cta - 1) / rows_cta;
+    pl.item_off[i] = static_cast<int>(items);
+    pl.merge_off[i] = static_cast<int>(merge);
+    items += static_cast<long long>(ns) * U.n_rb * Hkv;
+    if (ns > 1) {
+      pl.part_off[i] = part;
+      part += static_cast<long long>(ns) * Hkv * pl.G * U.T;
+      merge += static_cast<long long>(U.T) * Hq;
+    }
+  }
+  pl.item_off[B] = static_cast<int>(items);
+  pl.merge_off[B] = static_cast<int>(merge);
+  pl.n_items = static_cast<int>(items);
+  pl.n_merge = static_cast<int>(merge);
+  pl.part_rows = part;
+  pl.ws_bytes = part ? align_up(part * sizeof(float2), 256) + align_up(part * D * sizeof(float), 256) : 0;
+}
+
+template <int CAP>
+void fill_attn_params(AttnParams<CAP>& p, const AttnPlan& pl, const void* q, void* out, const int* bt,
+                      int max_blocks, float scale, unsigned* status, uint8_t* region) {
+  std::memset(&p, 0, sizeof(p));
+  p.q = static_cast<const __nv_bfloat16*>(q);
+  p.out = static_cast<__nv_bfloat16*>(out);
+  p.block_table = bt;
+  p.part_ml = reinterpret_cast<float2*>(region);
+  p.part_o = reinterpret_cast<float*>(region + align_up(pl.part_rows * sizeof(float2), 256));
+  p.status = status;
+  p.B = pl.B; p.Hq = pl.Hq; p.Hkv = pl.Hkv; p.G = pl.G; p.max_blocks = max_blocks;
+  p.n_items = pl.n_items; p.n_merge = pl.n_merge;
+  p.scale_log2 = scale * 1.4426950408889634f;
+  for (int i = 0; i <= pl.B; ++i) { p.item_off[i] = pl.item_off[i]; p.merge_off[i] = pl.merge_off[i]; }
+  for (int i = 0; i < pl.B; ++i) { p.part_off[i] = pl.part_off[i]; p.u[i] = pl.u[i]; }
+}
+
+template <int D, int NW, int CAP>
+int launch_attention_t(const AttnPlan& pl, const AttnParams<CAP>& p, const CUtensorMap& tk,
+                       const CUtensorMap& tv, cudaStream_t s, bool pdl) {
+  constexpr int STAGES = (D == 128) ? (NW == 4 ? 3 : 4) : 4;
+  auto kern = verify_attention_kernel<D, NW, STAGES, CAP>;
+  static std::mutex mu;
+  static bool attr_done[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return DIPSD_ERR_CUDA;
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    if (!attr_done[dev]) {
+      if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               static_cast<int>(attn_smem(D, STAGES))) != cudaSuccess)
+        return DIPSD_ERR_CUDA;
+      attr_done[dev] = true;
+    }
+  }
+  if (launch(kern, dim3(pl.n_items), dim3((NW + 1) * 32), attn_smem(D, STAGES), s, 0, pdl, p, tk, tv) !=
+      cudaSuccess)
+    return DIPSD_ERR_CUDA;
+  if (pl.n_merge > 0) {
+    auto mk = verify_attention_merge_kernel<D, CAP>;
+    if (launch(mk, dim3((pl.n_merge + 3) / 4), dim3(128), 0, s, 0, true, p) != cudaSuccess)
+      return DIPSD_ERR_CUDA;
+  }
+  return DIPSD_OK;
+}
+
+template <int CAP>
+int run_attention_cap(const AttnPlan& pl, const void* q, const void* kc, const void* vc, int num_blocks,
+                      const int* bt, int max_blocks, float scale, void* out, unsigned* status,
+                      uint8_t* region, cudaStream_t s, bool pdl) {
+  static thread_local AttnParams<CAP> p;
+  fill_attn_params<CAP>(p, pl, q, out, bt, max_blocks, scale, status, region);
+  alignas(64) CUtensorMap tk, tv;
+  if (!encode_cache_map(&tk, kc, num_blocks, pl.Hkv, pl.D) ||
+      !encode_cache_map(&tv, vc, num_blocks, pl.Hkv, pl.D))
+    return DIPSD_ERR_CUDA;
+  if (pl.D == 128)
+    return pl.NW == 4 ? launch_attention_t<128, 4, CAP>(pl, p, tk, tv, s, pdl)
+                      : launch_attention_t<128, 8, CAP>(pl, p, tk, tv, s, pdl);
+  return pl.NW == 4 ? launch_attention_t<64, 4, CAP>(pl, p, tk, tv, s, pdl)
+                    : launch_attention_t<64, 8, CAP>(pl, p, tk, tv, s, pdl);
+}
+
+int run_attention(const AttnPlan& pl, const void* q, const void* kc, const void* vc, int num_blocks,
+                  const int* bt, int max_blocks, float scale, void* out, unsigned* status, uint8_t* region,
+                  cudaStream_t s, bool pdl) {
+  if (pl.B <= kCapSmall)
+    return run_attention_cap<kCapSmall>(pl, q, kc, vc, num_blocks, bt, max_blocks, scale, out, status,
+                                        region, s, pdl);
+  return run_attention_cap<kCapLarge>(pl, q, kc, vc, num_blocks, bt, max_blocks, scale, out, status,
+                                      region, s, pdl);
+}
+
+int check_attn_buffers(const void* q, const void* kc, const void* vc, int num_blocks, const int* bt,
+                       int max_blocks, const void* out, int B, const int* L, const int* ctx, float scale) {
+  if (!q || !kc || !vc || !bt || !out) return DIPSD_ERR_INVALID_ARG;
+  if (!aligned(q, 16) || !aligned(kc, 16) || !aligned(vc, 16) || !aligned(out, 16) || !aligned(bt, 4))
+    return DIPSD_ERR_INVALID_ARG;
+  if (num_blocks < 1 || max_blocks < 1 || !std::isfinite(scale)) return DIPSD_ERR_INVALID_ARG;
+  if (q == out) return DIPSD_ERR_INVALID_ARG;
+  for (int i = 0; i < B; ++i)
+    if (static_cast<long long>(ctx[i]) + L[i] + 1 > static_cast<long long>(kPage) * max_blocks)
+      return DIPSD_ERR_INVALID_ARG;
+  return DIPSD_OK;
+}
+
+// ===================================================================== spec
+struct SpecPlan {
+  int B = 0, V = 0, vec = 1, nvec = 0, cl1 = 1, cl2 = 1;
+  int sum_t = 0, sum_l = 0;
+  std::vector<int> q_off, l_off;
+  size_t ws_bytes = 0;  // spec region only
+};
+
+int check_spec_users(int B, const int* L, int V) {
+  if (B < 1 || B > kMaxUsers || !L || V < 1) return DIPSD_ERR_INVALID_ARG;
+  long long st = 0;
+  for (int i = 0; i < B; ++i) {
+    if (L[i] < 0 || L[i] > kMaxDraft) return DIPSD_ERR_INVALID_ARG;
+    st += L[i] + 1;
+  }
+  if (st * static_cast<long long>(V) > (1ll << 40)) return DIPSD_ERR_INVALID_ARG;
+  return DIPSD_OK;
+}
+
+int cluster_for(int nvec) { return std::max(1, std::min(kMaxCluster, (nvec + 2047) / 2048)); }
+
+void plan_spec(int B, const int* L, int V, int elem, bool vec_ok, SpecPlan& pl) {
+  pl.B = B; pl.V = V;
+  pl.vec = vec_ok ? 16 / elem : 1;
+  pl.nvec = V / pl.vec;
+  pl.cl1 = cluster_for(pl.nvec);
+  pl.cl2 = cluster_for(pl.nvec);
+  pl.q_off.assign(B + 1, 0);
+  pl.l_off.assign(B + 1, 0);
+  for (int i = 0; i < B; ++i) {
+    pl.q_off[i + 1] = pl.q_off[i] + L[i] + 1;
+    pl.l_off[i + 1] = pl.l_off[i] + L[i];
+  }
+  pl.sum_t = pl.q_off[B];
+  pl.sum_l = pl.l_off[B];
+  pl.ws_bytes = align_up(static_cast<size_t>(pl.sum_t) * sizeof(float4), 256) + align_up(pl.sum_t, 256);
+}
+
+template <typename T, int VEC, int CAP>
+int launch_spec_t(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s, bool pdl) {
+  if (launch(spec_stats_kernel<T, VEC, CAP>, dim3(pl.sum_t * pl.cl1), dim3(kSpecThreads), 0, s, pl.cl1, pdl,
+             p) != cudaSuccess)
+    return DIPSD_ERR_CUDA;
+  if (launch(spec_sample_kernel<T, VEC, CAP>, dim3(pl.B * pl.cl2), dim3(kSpecThreads), 0, s, pl.cl2, true,
+             p) != cudaSuccess)
+    return DIPSD_ERR_CUDA;
+  return DIPSD_OK;
+}
+
+template <int CAP>
+int run_spec_cap(const SpecPlan& pl, int dtype, const void* z, const void* w, const int* dt, const float* uni,
+                 int* acc, int* offs, int* toks, float* probs, unsigned* status, uint8_t* region,
+                 cudaStream_t s, bool pdl) {
+  static thread_local SpecParams<CAP> p;
+  std::memset(&p, 0, sizeof(p));
+  p.z = z; p.w = w; p.draft_tokens = dt; p.uniforms = uni;
+  p.stats = reinterpret_cast<float4*>(region);
+  p.flags = region + align_up(static_cast<size_t>(pl.sum_t) * sizeof(float4), 256);
+  p.draft_probs = probs; p.accept_len = acc; p.out_offsets = offs; p.out_tokens = toks;
+  p.status = status;
+  p.B = pl.B; p.V = pl.V; p.nvec = pl.nvec;
+  for (int i = 0; i <= pl.B; ++i) { p.q_off[i] = pl.q_off[i]; p.l_off[i] = pl.l_off[i]; }
+  if (dtype == DIPSD_BF16)
+    return pl.vec == 8 ? launch_spec_t<__nv_bfloat16, 8, CAP>(pl, p, s, pdl)
+                       : launch_spec_t<__nv_bfloat16, 1, CAP>(pl, p, s, pdl);
+  return pl.vec == 4 ? launch_spec_t<float, 4, CAP>(pl, p, s, pdl) : launch_spec_t<float, 1, CAP>(pl, p, s, pdl);
+}
+
+int run_spec(const SpecPlan& pl, int dtype, const void* z, const void* w, const int* dt, const float* uni,
+             int* acc, int* offs, int* toks, float* probs, unsigned* status, uint8_t* region, cudaStream_t s,
+             bool pdl) {
+  if (pl.B <= kCapSmall)
+    return run_spec_cap<kCapSmall>(pl, dtype, z, w, dt, uni, acc, offs, toks, probs, status, region, s, pdl);
+  return run_spec_cap<kCapLarge>(pl, dtype, z, w, dt, uni, acc, offs, toks, probs, status, region, s, pdl);
+}
+
+int check_spec_buffers(int dtype, const void* z, const void* w, const int* dt, const float* uni, int* acc,
+                       int* offs, int* toks, float* probs, int sum_l, int V, bool* vec_ok) {
+  if (dtype != DIPSD_BF16 && dtype != DIPSD_F32) return DIPSD_ERR_INVALID_ARG;
+  if (!z || !uni || !acc || !offs || !toks) return DIPSD_ERR_INVALID_ARG;
+  if (sum_l > 0 && (!w || !dt)) return DIPSD_ERR_INVALID_ARG;
+  const size_t elem = dtype == DIPSD_BF16 ? 2 : 4;
+  if (!aligned(z, elem) || (w && !aligned(w, elem)) || !aligned(uni, 8) || !aligned(acc, 4) ||
+      !aligned(offs, 4) || !aligned(toks, 4) || (probs && !aligned(probs, 8)) || (dt && !aligned(dt, 4)))
+    return DIPSD_ERR_INVALID_ARG;
+  *vec_ok = (static_cast<size_t>(V) * elem) % 16 == 0 && aligned(z, 16) && (!w || aligned(w, 16));
+  return DIPSD_OK;
+}
+
+int check_workspace(const void* ws, size_t have, size_t need) {
+  if (!ws || !aligned(ws, 256) || have < need) return DIPSD_ERR_WORKSPACE;
+  return DIPSD_OK;
+}
+
+int cuda_status() { return cudaGetLastError() == cudaSuccess ? DIPSD_OK : DIPSD_ERR_CUDA; }
+
+}  // namespace
+}  // namespace dipsd
+
+using namespace dipsd;
+
+extern "C" {
+
+const char* dipsd_status_string(int status) {
+  switch (status) {
+    case DIPSD_OK: return "ok";
+    case DIPSD_ERR_INVALID_ARG: return "invalid argument";
+    case DIPSD_ERR_UNSUPPORTED: return "unsupported configuration";
+    case DIPSD_ERR_CUDA: return "CUDA error";
+    case DIPSD_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+    default: return "unknown status";
+  }
+}
+
+int dipsd_abi_version(void) { return DIPSD_ABI_VERSION; }
+
+long long dipsd_launch_count(void) { return g_launches; }
+
+size_t dipsd_verify_attention_workspace_size(int B, const int* h_L, const int* h_ctx, int Hq, int Hkv, int D) {
+  if (check_attn_users(B, h_L, h_ctx, Hq, Hkv, D) != DIPSD_OK) return 0;
+  DeviceFacts f;
+  if (!device_facts(f)) return 0;
+  AttnPlan pl;
+  plan_attention(B, h_L, h_ctx, nullptr, Hq, Hkv, D, f.sms, pl);
+  return kStatusBytes + pl.ws_bytes;
+}
+
+int dipsd_verify_attention(int B, const int* h_L, const int* h_ctx, const void* d_q, const void* d_k_cache,
+                           const void* d_v_cache, int num_blocks, const int* d_block_table, int max_blocks,
+                           int Hq, int Hkv, int D, float softmax_scale, void* d_out, void* d_workspace,
+                           size_t workspace_bytes, void* stream) {
+  int st = check_attn_users(B, h_L, h_ctx, Hq, Hkv, D);
+  if (st != DIPSD_OK) return st;
+  st = check_attn_buffers(d_q, d_k_cache, d_v_cache, num_blocks, d_block_table, max_blocks, d_out, B, h_L,
+                          h_ctx, softmax_scale);
+  if (st != DIPSD_OK) return st;
+  DeviceFacts f;
+  if (!device_facts(f)) return DIPSD_ERR_CUDA;
+  AttnPlan pl;
+  plan_attention(B, h_L, h_ctx, nullptr, Hq, Hkv, D, f.sms, pl);
+  st = check_workspace(d_workspace, workspace_bytes, kStatusBytes + pl.ws_bytes);
+  if (st != DIPSD_OK) return st;
+  uint8_t* ws = static_cast<uint8_t*>(d_workspace);
+  st = run_attention(pl, d_q, d_k_cache, d_v_cache, num_blocks, d_block_table, max_blocks, softmax_scale, d_out,
+                     reinterpret_cast<unsigned*>(ws), ws + kStatusBytes, static_cast<cudaStream_t>(stream), true);
+  return st != DIPSD_OK ? st : cuda_status();
+}
+
+size_t dipsd_spec_verify_workspace_size(int B, const int* h_L, int V) {
+  if (check_spec_users(B, h_L, V) != DIPSD_OK) return 0;
+  SpecPlan pl;
+  plan_spec(B, h_L, V, 2, false, pl);
+  return kStatusBytes + pl.ws_bytes;
+}
+
+int dipsd_spec_verify(int B, const int* h_L, int V, int logit_dtype, const void* d_target_logits,
+                      const void* d_draft_logits, const int* d_draft_tokens, const float* d_uniforms,
+                      int* d_accept_len, int* d_out_offsets, int* d_out_tokens, float* d_draft_probs,
+                      void* d_workspace, size_t workspace_bytes, void* stream) {
+  int st = check_spec_users(B, h_L, V);
+  if (st != DIPSD_OK) return st;
+  long long sum_l = 0;
+  for (int i = 0; i < B; ++i) sum_l += h_L[i];
+  bool vec_ok = false;
+  st = check_spec_buffers(logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
+                          d_out_offsets, d_out_tokens, d_draft_probs, static_cast<int>(sum_l), V, &vec_ok);
+  if (st != DIPSD_OK) return st;
+  SpecPlan pl;
+  plan_spec(B, h_L, V, logit_dtype == DIPSD_BF16 ? 2 : 4, vec_ok, pl);
+  st = check_workspace(d_workspace, workspace_bytes, kStatusBytes + pl.ws_bytes);
+  if (st != DIPSD_OK) return st;
+  uint8_t* ws = static_cast<uint8_t*>(d_workspace);
+  st = run_spec(pl, logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
+                d_out_offsets, d_out_tokens, d_draft_probs, reinterpret_cast<unsigned*>(ws), ws + kStatusBytes,
+                static_cast<cudaStream_t>(stream), true);
+  return st != DIPSD_OK ? st : cuda_status();
+}
+
+static int gather_members(int B, const int* members, int M, const int* L_all, const int* ctx_all,
+                          std::vector<int>& L, std::vector<int>& ctx) {
+  if (B < 1 || B > kMaxUsers || !members || M < 1 || !L_all || !ctx_all) return DIPSD_ERR_INVALID_ARG;
+  std::vector<char> seen(M, 0);
+  L.resize(B);
+  ctx.resize(B);
+  for (int b = 0; b < B; ++b) {
+    const int m = members[b];
+    if (m < 0 || m >= M || seen[m]) return DIPSD_ERR_INVALID_ARG;
+    seen[m] = 1;
+    L[b] = L_all[m];
+    ctx[b] = ctx_all[m];
+  }
+  return DIPSD_OK;
+}
+
+size_t dipsd_verify_batch_workspace_size(int B, const int* h_members, int M, const int* h_L_all,
+                                         const int* h_ctx_all, int Hq, int Hkv, int D, int V) {
+  std::vector<int> L, ctx;
+  if (gather_members(B, h_members, M, h_L_all, h_ctx_all, L, ctx) != DIPSD_OK) return 0;
+  if (check_attn_users(B, L.data(), ctx.data(), Hq, Hkv, D) != DIPSD_OK) return 0;
+  if (check_spec_users(B, L.data(), V) != DIPSD_OK) return 0;
+  DeviceFacts f;
+  if (!device_facts(f)) return 0;
+  AttnPlan ap;
+  plan_attention(B, L.data(), ctx.data(), h_members, Hq, Hkv, D, f.sms, ap);
+  SpecPlan sp;
+  plan_spec(B, L.data(), V, 2, false, sp);
+  return kStatusBytes + align_up(ap.ws_bytes, 256) + sp.ws_bytes;
+}
+
+int dipsd_verify_batch(int B, const int* h_members, int M, const int* h_L_all, const int* h_ctx_all,
+                       const void* d_q, const void* d_k_cache, const void* d_v_cache, int num_blocks,
+                       const int* d_block_table_all, int max_blocks, int Hq, int Hkv, int D, float softmax_scale,
+                       void* d_attn_out, int V, int logit_dtype, const void* d_target_logits,
+                       const void* d_draft_logits, const int* d_draft_tokens, const float* d_uniforms,
+                       int* d_accept_len, int* d_out_offsets, int* d_out_tokens, float* d_draft_probs,
+                       void* d_workspace, size_t workspace_bytes, void* stream) {
+  std::vector<int> L, ctx;
+  int st = gather_members(B, h_members, M, h_L_all, h_ctx_all, L, ctx);
+  if (st != DIPSD_OK) return st;
+  st = check_attn_users(B, L.data(), ctx.data(), Hq, Hkv, D);
+  if (st != DIPSD_OK) return st;
+  st = check_spec_users(B, L.data(), V);
+  if (st != DIPSD_OK) return st;
+  st = check_attn_buffers(d_q, d_k_cache, d_v_cache, num_blocks, d_block_table_all, max_blocks, d_attn_out, B,
+                          L.data(), ctx.data(), softmax_scale);
+  if (st != DIPSD_OK) return st;
+  long long sum_l = 0;
+  for (int b = 0; b < B; ++b) sum_l += L[b];
+  bool vec_ok = false;
+  st = check_spec_buffers(logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
+                          d_out_offsets, d_out_tokens, d_draft_probs, static_cast<int>(sum_l), V, &vec_ok);
+  if (st != DIPSD_OK) return st;
+  DeviceFacts f;
+  if (!device_facts(f)) return DIPSD_ERR_CUDA;
+  AttnPlan ap;
+  plan_attention(B, L.data(), ctx.data(), h_members, Hq, Hkv, D, f.sms, ap);
+  SpecPlan sp;
+  plan_spec(B, L.data(), V, logit_dtype == DIPSD_BF16 ? 2 : 4, vec_ok, sp);
+  const size_t attn_region = align_up(ap.ws_bytes, 256);
+  st = check_workspace(d_workspace, workspace_bytes, kStatusBytes + attn_region + sp.ws_bytes);
+  if (st != DIPSD_OK) return st;
+  uint8_t* ws = static_cast<uint8_t*>(d_workspace);
+  unsigned* status = reinterpret_cast<unsigned*>(ws);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  st = run_attention(ap, d_q, d_k_cache, d_v_cache, num_blocks, d_block_table_all, max_blocks, softmax_scale,
+                     d_attn_out, status, ws + kStatusBytes, s, true);
+  if (st != DIPSD_OK) return st;
+  st = run_spec(sp, logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
+                d_out_offsets, d_out_tokens, d_draft_probs, status, ws + kStatusBytes + attn_region, s, true);
+  return st != DIPSD_OK ? st : cuda_status();
+}
+
+}  // extern "C"

@@ -1,0 +1,257 @@
+"""Python binding of libdipsd.so (the C ABI in include/dipsd.h).
+
+Argument marshalling only: every step of verification runs in the library's
+CUDA kernels.  Functions carry the C names; tensors are torch CUDA tensors
+(device memory and streams come from PyTorch), per-user lengths are host
+sequences.  If the library is missing this module raises instead of falling
+back to anything else.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Sequence
+
+import numpy as np
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libdipsd.so")
+
+DIPSD_OK = 0
+DIPSD_BF16 = 0
+DIPSD_F32 = 1
+PAGE_SIZE = 16
+MAX_USERS = 512
+MAX_DRAFT = 31
+DEVERR_WAIT_TIMEOUT = 1
+DEVERR_BAD_TOKEN = 2
+
+EXPORTS = (
+    "dipsd_status_string", "dipsd_abi_version", "dipsd_launch_count",
+    "dipsd_verify_attention_workspace_size", "dipsd_verify_attention",
+    "dipsd_spec_verify_workspace_size", "dipsd_spec_verify",
+    "dipsd_verify_batch_workspace_size", "dipsd_verify_batch",
+)
+
+_lib: Optional[ctypes.CDLL] = None
+_i32p = ctypes.POINTER(ctypes.c_int)
+_vp = ctypes.c_void_p
+_sz = ctypes.c_size_t
+_i = ctypes.c_int
+
+
+class DipsdError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        super().__init__(f"{where}: {status_string(status)} (status {status})")
+        self.status = status
+
+
+def load(path: str = LIB_PATH) -> ctypes.CDLL:
+    """Loads the library once; raises if it has not been built."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is missing: build it with __graft_entry__.build()")
+    lib = ctypes.CDLL(path)
+    lib.dipsd_status_string.restype = ctypes.c_char_p
+    lib.dipsd_status_string.argtypes = [_i]
+    lib.dipsd_abi_version.restype = _i
+    lib.dipsd_launch_count.restype = ctypes.c_longlong
+    lib.dipsd_verify_attention_workspace_size.restype = _sz
+    lib.dipsd_verify_attention_workspace_size.argtypes = [_i, _i32p, _i32p, _i, _i, _i]
+    lib.dipsd_verify_attention.restype = _i
+    lib.dipsd_verify_attention.argtypes = [_i, _i32p, _i32p, _vp, _vp, _vp, _i, _vp, _i, _i, _i, _i,
+                                           ctypes.c_float, _vp, _vp, _sz, _vp]
+    lib.dipsd_spec_verify_workspace_size.restype = _sz
+    lib.dipsd_spec_verify_workspace_size.argtypes = [_i, _i32p, _i]
+    lib.dipsd_spec_verify.restype = _i
+    lib.dipsd_spec_verify.argtypes = [_i, _i32p, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
+    lib.dipsd_verify_batch_workspace_size.restype = _sz
+    lib.dipsd_verify_batch_workspace_size.argtypes = [_i, _i32p, _i, _i32p, _i32p, _i, _i, _i, _i]
+    lib.dipsd_verify_batch.restype = _i
+    lib.dipsd_verify_batch.argtypes = [_i, _i32p, _i, _i32p, _i32p, _vp, _vp, _vp, _i, _vp, _i, _i, _i, _i,
+                                       ctypes.c_float, _vp, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                       _vp, _sz, _vp]
+    _lib = lib
+    return lib
+
+
+def dipsd_launch_count() -> int:
+    """Kernels launched by the library from this host thread so far."""
+    return int(load().dipsd_launch_count())
+
+
+def status_string(status: int) -> str:
+    return load().dipsd_status_string(int(status)).decode()
+
+
+def _check(status: int, where: str) -> None:
+    if status != DIPSD_OK:
+        raise DipsdError(status, where)
+
+
+def _host_i32(x: Sequence[int]):
+    a = np.ascontiguousarray(np.asarray(x, dtype=np.int32))
+    return a, a.ctypes.data_as(_i32p)
+
+
+def _dptr(t: Optional[torch.Tensor], name: str, dtype=None) -> int:
+    if t is None:
+        return 0
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    return t.data_ptr()
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def _logit_dtype(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return DIPSD_BF16
+    if t.dtype == torch.float32:
+        return DIPSD_F32
+    raise ValueError(f"logits must be bf16 or fp32, got {t.dtype}")
+
+
+def workspace(nbytes: int, device) -> torch.Tensor:
+    """Zero-filled device buffer usable as a workspace (status word starts at 0)."""
+    return torch.zeros(max(int(nbytes), 256), dtype=torch.uint8, device=device)
+
+
+def device_status(ws: torch.Tensor) -> int:
+    """Device status word (DEVERR_* bits) of a workspace; synchronises on its stream."""
+    return int(ws[:4].view(torch.int32).item())
+
+
+# ---------------------------------------------------------------- attention
+def dipsd_verify_attention_workspace_size(L, ctx, Hq: int, Hkv: int, D: int) -> int:
+    a, pa = _host_i32(L)
+    b, pb = _host_i32(ctx)
+    return int(load().dipsd_verify_attention_workspace_size(len(a), pa, pb, Hq, Hkv, D))
+
+
+def dipsd_verify_attention(L, ctx, q, k_cache, v_cache, block_table, softmax_scale: float, out=None,
+                           ws=None, stream=None) -> torch.Tensor:
+    """Causal GQA attention of every verify token over its user's paged KV cache."""
+    lib = load()
+    a, pa = _host_i32(L)
+    b, pb = _host_i32(ctx)
+    sum_t = int((a + 1).sum())
+    nb, Hkv, page, D = k_cache.shape
+    Hq = q.shape[1]
+    if page != PAGE_SIZE or tuple(q.shape) != (sum_t, Hq, D) or tuple(v_cache.shape) != tuple(k_cache.shape):
+        raise ValueError("shape mismatch between q, caches and lengths")
+    if block_table.dim() != 2 or block_table.shape[0] != len(a):
+        raise ValueError("block_table must be [B][max_blocks]")
+    if out is None:
+        out = torch.empty_like(q)
+    if ws is None:
+        ws = workspace(dipsd_verify_attention_workspace_size(a, b, Hq, Hkv, D), q.device)
+    st = lib.dipsd_verify_attention(len(a), pa, pb, _dptr(q, "q", torch.bfloat16),
+                                    _dptr(k_cache, "k_cache", torch.bfloat16),
+                                    _dptr(v_cache, "v_cache", torch.bfloat16), nb,
+                                    _dptr(block_table, "block_table", torch.int32), block_table.shape[1],
+                                    Hq, Hkv, D, float(softmax_scale), _dptr(out, "out", torch.bfloat16),
+                                    _dptr(ws, "workspace"), ws.numel(), _stream(stream))
+    _check(st, "dipsd_verify_attention")
+    return out
+
+
+# ---------------------------------------------------------- spec verification
+def dipsd_spec_verify_workspace_size(L, V: int) -> int:
+    a, pa = _host_i32(L)
+    return int(load().dipsd_spec_verify_workspace_size(len(a), pa, V))
+
+
+def spec_outputs(L, device, with_probs=True):
+    """Output tensors of one spec-verify call: accept_len, out_offsets, out_tokens, draft_probs."""
+    B = len(L)
+    sum_t = int(np.asarray(L).sum()) + B
+    return (torch.empty(B, dtype=torch.int32, device=device),
+            torch.empty(B + 1, dtype=torch.int32, device=device),
+            torch.empty(sum_t, dtype=torch.int32, device=device),
+            torch.empty(sum_t, 2, dtype=torch.float32, device=device) if with_probs else None)
+
+
+def dipsd_spec_verify(L, target_logits, draft_logits, draft_tokens, uniforms, outputs=None, ws=None,
+                      stream=None):
+    """Speculative verification; returns (accept_len, out_offsets, out_tokens, draft_probs)."""
+    lib = load()
+    a, pa = _host_i32(L)
+    sum_t, sum_l = int((a + 1).sum()), int(a.sum())
+    V = target_logits.shape[1]
+    dt = _logit_dtype(target_logits)
+    if target_logits.shape[0] != sum_t or tuple(uniforms.shape) != (sum_t, 2):
+        raise ValueError("target_logits / uniforms do not match the draft lengths")
+    if draft_logits.shape != (sum_l, V) or draft_logits.dtype != target_logits.dtype or draft_tokens.numel() != sum_l:
+        raise ValueError("draft_logits / draft_tokens do not match the draft lengths")
+    acc, offs, toks, probs = outputs if outputs is not None else spec_outputs(a, target_logits.device)
+    if ws is None:
+        ws = workspace(dipsd_spec_verify_workspace_size(a, V), target_logits.device)
+    st = lib.dipsd_spec_verify(len(a), pa, V, dt, _dptr(target_logits, "target_logits"),
+                               _dptr(draft_logits, "draft_logits") if sum_l else 0,
+                               _dptr(draft_tokens, "draft_tokens", torch.int32) if sum_l else 0,
+                               _dptr(uniforms, "uniforms", torch.float32),
+                               _dptr(acc, "accept_len", torch.int32), _dptr(offs, "out_offsets", torch.int32),
+                               _dptr(toks, "out_tokens", torch.int32),
+                               _dptr(probs, "draft_probs", torch.float32), _dptr(ws, "workspace"), ws.numel(),
+                               _stream(stream))
+    _check(st, "dipsd_spec_verify")
+    return acc, offs, toks, probs
+
+
+# ---------------------------------------------------------------- one stage
+def dipsd_verify_batch_workspace_size(members, L_all, ctx_all, Hq, Hkv, D, V) -> int:
+    m, pm = _host_i32(members)
+    a, pa = _host_i32(L_all)
+    b, pb = _host_i32(ctx_all)
+    return int(load().dipsd_verify_batch_workspace_size(len(m), pm, len(a), pa, pb, Hq, Hkv, D, V))
+
+
+def dipsd_verify_batch(members, L_all, ctx_all, q, k_cache, v_cache, block_table_all, softmax_scale,
+                       target_logits, draft_logits, draft_tokens, uniforms, attn_out=None, outputs=None,
+                       ws=None, stream=None):
+    """Attention then speculative verification for the users `members` of one stage.
+
+    Returns (attn_out, accept_len, out_offsets, out_tokens, draft_probs).
+    """
+    lib = load()
+    m, pm = _host_i32(members)
+    a, pa = _host_i32(L_all)
+    b, pb = _host_i32(ctx_all)
+    Lb = a[m]
+    sum_t, sum_l = int((Lb + 1).sum()), int(Lb.sum())
+    nb, Hkv, page, D = k_cache.shape
+    Hq, V = q.shape[1], target_logits.shape[1]
+    if page != PAGE_SIZE or tuple(q.shape) != (sum_t, Hq, D):
+        raise ValueError("q does not match the members' draft lengths")
+    if target_logits.shape[0] != sum_t or draft_logits.shape != (sum_l, V) or tuple(uniforms.shape) != (sum_t, 2):
+        raise ValueError("logits / uniforms do not match the members' draft lengths")
+    if attn_out is None:
+        attn_out = torch.empty_like(q)
+    acc, offs, toks, probs = outputs if outputs is not None else spec_outputs(Lb, q.device)
+    if ws is None:
+        ws = workspace(dipsd_verify_batch_workspace_size(m, a, b, Hq, Hkv, D, V), q.device)
+    st = lib.dipsd_verify_batch(len(m), pm, len(a), pa, pb, _dptr(q, "q", torch.bfloat16),
+                                _dptr(k_cache, "k_cache", torch.bfloat16), _dptr(v_cache, "v_cache", torch.bfloat16),
+                                nb, _dptr(block_table_all, "block_table", torch.int32), block_table_all.shape[1],
+                                Hq, Hkv, D, float(softmax_scale), _dptr(attn_out, "attn_out", torch.bfloat16), V,
+                                _logit_dtype(target_logits), _dptr(target_logits, "target_logits"),
+                                _dptr(draft_logits, "draft_logits") if sum_l else 0,
+                                _dptr(draft_tokens, "draft_tokens", torch.int32) if sum_l else 0,
+                                _dptr(uniforms, "uniforms", torch.float32),
+                                _dptr(acc, "accept_len", torch.int32), _dptr(offs, "out_offsets", torch.int32),
+                                _dptr(toks, "out_tokens", torch.int32), _dptr(probs, "draft_probs", torch.float32),
+                                _dptr(ws, "workspace"), ws.numel(), _stream(stream))
+    _check(st, "dipsd_verify_batch")
+    return attn_out, acc, offs, toks, probs

@@ -1,0 +1,94 @@
+"""Shared comparison logic for the GPU parity tests (CUDA path vs oracle).
+
+Tolerances (stated by the task's acceptance bar):
+  * attention: |gpu - oracle| <= 2e-2 absolute or <= 1e-2 relative, per element;
+  * probabilities p_t(d), q_t(d): within 1e-5 absolute;
+  * accept lengths, emitted tokens, offsets: bit-exact, except for users with a
+    decision whose uniform lies within 1e-6 of the acceptance ratio or of a
+    CDF edge of the sampled token; those are counted and must stay under 1e-4
+    of the positions.
+"""
+import numpy as np
+import torch
+
+import oracle
+from workloads import offsets
+
+ATOL, RTOL = 2e-2, 1e-2
+PROB_ATOL = 1e-5
+BAND = 1e-6
+
+
+def attention_subset_reference(b, users):
+    """Oracle output rows for the chosen batch users (pages copied to the host)."""
+    users = np.asarray(users)
+    qo = offsets(b.T)
+    rows = np.concatenate([np.arange(qo[i], qo[i + 1]) for i in users])
+    bt_all = b.block_table.cpu().numpy()
+    bt = bt_all[b.members[users]].astype(np.int64)
+    used = []
+    for k, i in enumerate(users):
+        n = -(-int(b.kv_len[i]) // 16)
+        used.append(bt[k, :n])
+    need = np.unique(np.concatenate(used))
+    remap = {int(x): j for j, x in enumerate(need)}
+    bt2 = np.full_like(bt, -1)
+    for k, i in enumerate(users):
+        n = -(-int(b.kv_len[i]) // 16)
+        bt2[k, :n] = [remap[int(x)] for x in bt[k, :n]]
+    idx = torch.from_numpy(need).to(b.k_cache.device)
+    kc = b.k_cache.index_select(0, idx).double().cpu().numpy()
+    vc = b.v_cache.index_select(0, idx).double().cpu().numpy()
+    q = b.q.cpu()[torch.from_numpy(rows)].double().numpy()
+    ref = oracle.verify_attention(q, kc, vc, bt2, b.ctx[users], b.L[users], b.scale)
+    return rows, ref
+
+
+def check_attention(out, ref):
+    got = out.double().cpu().numpy() if torch.is_tensor(out) else out
+    err = np.abs(got - ref)
+    ok = (err <= ATOL) | (err <= RTOL * np.abs(ref))
+    assert np.isfinite(got).all(), "non-finite attention output"
+    assert ok.all(), f"attention mismatch: {(~ok).sum()} elements, max err {err.max():.3e}"
+    return float(err.max())
+
+
+def spec_reference(b):
+    return oracle.spec_verify(b.L, b.target_logits.double().cpu().numpy(), b.draft_logits.double().cpu().numpy(),
+                              b.draft_tokens.cpu().numpy(), b.uniforms.cpu().numpy())
+
+
+def check_spec(b, acc, offs, toks, probs, ref=None):
+    """Compares one spec-verify result with the oracle; returns counters."""
+    ref = spec_reference(b) if ref is None else ref
+    acc = acc.cpu().numpy().astype(np.int64)
+    offs = offs.cpu().numpy().astype(np.int64)
+    toks = toks.cpu().numpy().astype(np.int64)
+    B = b.B
+    # packing is self-consistent and exact
+    assert offs[0] == 0 and np.all(np.diff(offs) == acc + 1)
+    assert np.all(acc >= 0) and np.all(acc <= b.L)
+    qo, lo = offsets(b.T), offsets(b.L)
+    dt = b.draft_tokens.cpu().numpy()
+    if probs is not None:
+        pr = probs.cpu().numpy()
+        draft_pos = np.concatenate([np.arange(qo[i], qo[i] + b.L[i]) for i in range(B)] + [np.zeros(0, int)])
+        bonus_pos = qo[1:] - 1
+        np.testing.assert_allclose(pr[draft_pos, 0], ref["p_d"][draft_pos], atol=PROB_ATOL, rtol=0)
+        np.testing.assert_allclose(pr[draft_pos, 1], ref["q_d"][draft_pos], atol=PROB_ATOL, rtol=0)
+        assert np.all(pr[bonus_pos] == 0)
+    near = oracle.decision_margins(ref, b.L, BAND)
+    for i in range(B):
+        seg = toks[offs[i]:offs[i + 1]]
+        np.testing.assert_array_equal(seg[:acc[i]], dt[lo[i]:lo[i] + acc[i]])
+        assert 0 <= seg[-1] < b.V
+        if near[i]:
+            continue
+        assert acc[i] == ref["accept_len"][i], (i, acc[i], ref["accept_len"][i])
+        rseg = ref["out_tokens"][ref["out_offsets"][i]:ref["out_offsets"][i + 1]]
+        np.testing.assert_array_equal(seg, rseg, err_msg=f"user {i}")
+    positions = int(b.T.sum())
+    n_near = int(near.sum())
+    assert n_near <= 1e-4 * positions, f"{n_near} near-boundary users out of {positions} positions"
+    return dict(users=B, positions=positions, near=n_near,
+                emitted=int(offs[-1]), mean_accept=float(acc.mean()))

@@ -1,0 +1,75 @@
+"""dipsd_verify_batch (one pipeline stage's users) vs the oracle, incl. the
+pipelined schedule of four stages on two streams."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from parity import attention_subset_reference, check_attention, check_spec
+from workloads import make_config
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+
+
+def _launch(dipsd, b, L_all, ctx_all, kc, vc, bt, stream):
+    g = lambda t: t.to(DEV, non_blocking=True)
+    with torch.cuda.stream(stream):
+        res = dipsd.dipsd_verify_batch(b.members, L_all, ctx_all, g(b.q), kc, vc, bt, b.scale,
+                                       g(b.target_logits), g(b.draft_logits), g(b.draft_tokens),
+                                       g(b.uniforms), stream=stream)
+    return res
+
+
+def test_pipelined_stages_on_two_streams(cuda_lib):
+    """Workload 5: 128 users dealt into 4 batches of 32, verified back to back on two streams."""
+    batches = make_config(5, seed=0, device="cpu", kv_device=DEV)
+    from workloads import config_shape
+    s = config_shape(5)
+    L_all, ctx_all = s["L"], s["ctx"]
+    kc, vc = batches[0].k_cache, batches[0].v_cache
+    bt = batches[0].block_table.to(DEV)
+    streams = [torch.cuda.Stream(), torch.cuda.Stream()]
+    results = [_launch(cuda_lib, b, L_all, ctx_all, kc, vc, bt, streams[n % 2]) for n, b in enumerate(batches)]
+    torch.cuda.synchronize()
+    for n, (b, (attn, acc, offs, toks, probs)) in enumerate(zip(batches, results)):
+        st = check_spec(b, acc, offs, toks, probs)
+        users = [0, int(np.argmax(b.ctx)), b.B - 1]
+        rows, ref = attention_subset_reference(b, users)
+        err = check_attention(attn[torch.from_numpy(rows).to(DEV)], ref)
+        print(f"stage {n}: {st}, attention max err {err:.3e}")
+
+
+def test_batch_matches_separate_calls(cuda_lib):
+    b = make_config(2, seed=4)
+    g = lambda t: t.to(DEV)
+    q, kc, vc, bt = g(b.q), g(b.k_cache), g(b.v_cache), g(b.block_table)
+    z, w, d, u = g(b.target_logits), g(b.draft_logits), g(b.draft_tokens), g(b.uniforms)
+    attn_a = cuda_lib.dipsd_verify_attention(b.L, b.ctx, q, kc, vc, bt, b.scale)
+    sv = cuda_lib.dipsd_spec_verify(b.L, z, w, d, u)
+    res = cuda_lib.dipsd_verify_batch(b.members, b.L, b.ctx, q, kc, vc, bt, b.scale, z, w, d, u)
+    torch.cuda.synchronize()
+    assert torch.equal(attn_a, res[0])
+    for x, y in zip(sv, res[1:]):
+        assert torch.equal(x, y)
+
+
+def test_batch_with_permuted_membership(cuda_lib):
+    """Members name rows of a larger user table, in any order."""
+    b = make_config(1, seed=5)
+    # table of 6 users: batch users sit at rows 4, 0, 5, 2
+    perm = np.array([4, 0, 5, 2])
+    L_all = np.zeros(6, np.int32)
+    ctx_all = np.zeros(6, np.int32)
+    L_all[perm], ctx_all[perm] = b.L, b.ctx
+    bt_all = torch.full((6, b.block_table.shape[1]), -1, dtype=torch.int32)
+    bt_all[torch.from_numpy(perm)] = b.block_table
+    g = lambda t: t.to(DEV)
+    attn, acc, offs, toks, probs = cuda_lib.dipsd_verify_batch(
+        perm, L_all, ctx_all, g(b.q), g(b.k_cache), g(b.v_cache), g(bt_all), b.scale, g(b.target_logits),
+        g(b.draft_logits), g(b.draft_tokens), g(b.uniforms))
+    torch.cuda.synchronize()
+    ref = oracle.verify_attention(b.q.double().numpy(), b.k_cache.double().numpy(), b.v_cache.double().numpy(),
+                                  b.block_table.numpy(), b.ctx, b.L, b.scale)
+    check_attention(attn, ref)
+    check_spec(b, acc, offs, toks, probs)

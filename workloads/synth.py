@@ -189,8 +189,12 @@ def make_spec_inputs(rng, L, user_ids, V, logit_std, noise_sigma, logit_dtype, s
 
 def make_batch(L, ctx, *, Hq, Hkv, D, V, logit_std=1.0, noise_sigma=1.0,
                logit_dtype="bf16", seed=0, device="cpu", kv_device=None,
-               alpha=None, spare_pages=3, user_ids=None) -> Batch:
-    """Build one batch from explicit per-user draft and context lengths."""
+               alpha=None, spare_pages=3, user_ids=None, spec_only=False) -> Batch:
+    """Build one batch from explicit per-user draft and context lengths.
+
+    spec_only=True skips the KV cache, block table and Q (the speculative
+    sampling inputs are identical either way).
+    """
     L = np.asarray(L, dtype=np.int32)
     ctx = np.asarray(ctx, dtype=np.int32)
     B = int(L.shape[0])
@@ -198,9 +202,12 @@ def make_batch(L, ctx, *, Hq, Hkv, D, V, logit_std=1.0, noise_sigma=1.0,
     rng = np.random.default_rng([seed, 1])
     kv_len = ctx + L + 1
     bt, num_blocks = _block_tables(rng, kv_len, spare_pages)
-    k_cache = _randn_bf16((num_blocks, Hkv, PAGE, D), seed * 7919 + 11, kv_device)
-    v_cache = _randn_bf16((num_blocks, Hkv, PAGE, D), seed * 7919 + 13, kv_device)
-    q = _randn_bf16((int((L + 1).sum()), Hq, D), seed * 7919 + 17, "cpu").to(device)
+    if spec_only:
+        k_cache = v_cache = q = None
+    else:
+        k_cache = _randn_bf16((num_blocks, Hkv, PAGE, D), seed * 7919 + 11, kv_device)
+        v_cache = _randn_bf16((num_blocks, Hkv, PAGE, D), seed * 7919 + 13, kv_device)
+        q = _randn_bf16((int((L + 1).sum()), Hq, D), seed * 7919 + 17, "cpu").to(device)
     uid = np.arange(B, dtype=np.int32) if user_ids is None else np.asarray(user_ids, np.int32)
     srng = np.random.default_rng([seed, 2])
     zt, wt, d, uni = make_spec_inputs(srng, L, uid, V, logit_std, noise_sigma, logit_dtype, seed)
@@ -263,14 +270,14 @@ def _ndtr(x):
     return 0.5 * math.erfc(-x / math.sqrt(2.0))
 
 
-def make_config(cfg: int, seed: int = 0, device="cpu", kv_device=None):
+def make_config(cfg: int, seed: int = 0, device="cpu", kv_device=None, spec_only=False):
     """Workload 1-4 as one Batch; workload 5 as a list of 4 Batches sharing one KV pool."""
     s = config_shape(cfg, seed)
     if cfg != 5:
         return make_batch(s["L"], s["ctx"], Hq=s["Hq"], Hkv=s["Hkv"], D=s["D"], V=s["V"],
                           logit_std=s["logit_std"], noise_sigma=s["noise_sigma"],
                           logit_dtype=s["logit_dtype"], seed=seed, device=device,
-                          kv_device=kv_device, alpha=s["alpha"])
+                          kv_device=kv_device, alpha=s["alpha"], spec_only=spec_only)
     return make_pipeline(s, seed, device, kv_device)
 
 
