@@ -5,8 +5,11 @@ Tolerances (stated by the task's acceptance bar):
   * probabilities p_t(d), q_t(d): within 1e-5 absolute;
   * accept lengths, emitted tokens, offsets: bit-exact, except for users with a
     decision whose uniform lies within 1e-6 of the acceptance ratio or of a
-    CDF edge of the sampled token; those are counted and must stay under 1e-4
-    of the positions.
+    CDF edge of the sampled token ("near-boundary", counted and reported).
+    A user whose output differs from the oracle must be near-boundary, and
+    such mismatches must stay under 1e-4 of the verify positions.  (Near-
+    boundary users themselves are common at V = 151936: the sampled token's
+    CDF cell is ~1e-5 wide, so the band catches a uniform in ~10% of users.)
 """
 import numpy as np
 import torch
@@ -78,17 +81,23 @@ def check_spec(b, acc, offs, toks, probs, ref=None):
         np.testing.assert_allclose(pr[draft_pos, 1], ref["q_d"][draft_pos], atol=PROB_ATOL, rtol=0)
         assert np.all(pr[bonus_pos] == 0)
     near = oracle.decision_margins(ref, b.L, BAND)
+    mismatch = np.zeros(B, dtype=bool)
     for i in range(B):
         seg = toks[offs[i]:offs[i + 1]]
         np.testing.assert_array_equal(seg[:acc[i]], dt[lo[i]:lo[i] + acc[i]])
         assert 0 <= seg[-1] < b.V
-        if near[i]:
-            continue
-        assert acc[i] == ref["accept_len"][i], (i, acc[i], ref["accept_len"][i])
         rseg = ref["out_tokens"][ref["out_offsets"][i]:ref["out_offsets"][i + 1]]
-        np.testing.assert_array_equal(seg, rseg, err_msg=f"user {i}")
+        mismatch[i] = acc[i] != ref["accept_len"][i] or not np.array_equal(seg, rseg)
     positions = int(b.T.sum())
-    n_near = int(near.sum())
-    assert n_near <= 1e-4 * positions, f"{n_near} near-boundary users out of {positions} positions"
-    return dict(users=B, positions=positions, near=n_near,
+    far = np.flatnonzero(mismatch & ~near)
+    assert far.size == 0, f"users {far.tolist()} differ from the oracle away from any decision boundary"
+    n_mis = int(mismatch.sum())
+    assert n_mis <= 1e-4 * positions, f"{n_mis} near-boundary mismatches out of {positions} positions"
+    return dict(users=B, positions=positions, near=int(near.sum()), mismatches=n_mis,
                 emitted=int(offs[-1]), mean_accept=float(acc.mean()))
+
+
+def valid_spec_outputs(acc, offs, toks, probs):
+    """The defined part of a spec-verify result (out_tokens past out_offsets[B] is capacity)."""
+    n = int(offs[-1].item())
+    return [acc, offs, toks[:n]] + ([probs] if probs is not None else [])
