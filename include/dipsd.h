@@ -170,6 +170,34 @@ int dipsd_verify_batch(int B, const int* h_members, int M,
                        int* d_out_tokens, float* d_draft_probs,
                        void* d_workspace, size_t workspace_bytes, void* stream);
 
+/* ------------------------------------------------------------------------
+ * Speculative verification without a caller-provided workspace.
+ *
+ * The paper has no counterpart to this entry point; it exists for callers
+ * that cannot allocate device memory themselves: for example a plugin inside
+ * a host program whose own pool owns all device memory, or a serving loop
+ * that must not call cudaMalloc because it can synchronise the device.  It
+ * computes exactly what dipsd_spec_verify computes, with the same arguments
+ * minus the workspace, and allocates nothing (no cudaMalloc, no cudaFree, no
+ * allocating library routine).
+ *
+ * Scratch lives in one static device array of the library, sized for at most
+ * DIPSD_NOALLOC_MAX_POSITIONS verify positions (sum_i (L_i+1)); a larger batch
+ * is rejected with DIPSD_ERR_UNSUPPORTED before anything is launched.  Every
+ * GPU that loads the library holds that array (about 70 KB) until the process
+ * exits.  The first call on a device looks up the array's device address with
+ * that device current; make that first call before any stream capture.  All
+ * calls share the one array: calls that overlap on the GPU (other streams,
+ * other host threads) race and must be serialised by the caller.  Each call
+ * clears the array's status word on `stream` before its kernels run.
+ * ---------------------------------------------------------------------- */
+#define DIPSD_NOALLOC_MAX_POSITIONS 4096
+int dipsd_spec_verify_noalloc(int B, const int* h_L, int V, int logit_dtype,
+                              const void* d_target_logits, const void* d_draft_logits,
+                              const int* d_draft_tokens, const float* d_uniforms,
+                              int* d_accept_len, int* d_out_offsets, int* d_out_tokens,
+                              float* d_draft_probs, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

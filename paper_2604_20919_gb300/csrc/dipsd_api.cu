@@ -405,8 +405,34 @@ int check_workspace(const void* ws, size_t have, size_t need) {
 
 int cuda_status() { return cudaGetLastError() == cudaSuccess ? DIPSD_OK : DIPSD_ERR_CUDA; }
 
+// ------------------------------------------------------- no-alloc scratch
+// Scratch of dipsd_spec_verify_noalloc: status word, per-position row
+// statistics and acceptance bits for up to DIPSD_NOALLOC_MAX_POSITIONS
+// positions, laid out exactly like a dipsd_spec_verify workspace.
+constexpr size_t kNoAllocScratchBytes =
+    kStatusBytes + ((DIPSD_NOALLOC_MAX_POSITIONS * sizeof(float4) + 255) / 256) * 256 +
+    ((DIPSD_NOALLOC_MAX_POSITIONS + 255) / 256) * 256;
+
 }  // namespace
 }  // namespace dipsd
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[dipsd::kNoAllocScratchBytes];
+
+// Device address of g_noalloc_scratch on the current device (looked up once
+// per device, with that device current); nullptr if the lookup fails.
+static uint8_t* noalloc_scratch() {
+  static std::mutex mu;
+  static void* addr[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> lock(mu);
+  if (!addr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess) return nullptr;
+    addr[dev] = p;
+  }
+  return static_cast<uint8_t*>(addr[dev]);
+}
 
 using namespace dipsd;
 
@@ -484,6 +510,35 @@ int dipsd_spec_verify(int B, const int* h_L, int V, int logit_dtype, const void*
   st = run_spec(pl, logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
                 d_out_offsets, d_out_tokens, d_draft_probs, reinterpret_cast<unsigned*>(ws), ws + kStatusBytes,
                 static_cast<cudaStream_t>(stream), true);
+  return st != DIPSD_OK ? st : cuda_status();
+}
+
+int dipsd_spec_verify_noalloc(int B, const int* h_L, int V, int logit_dtype, const void* d_target_logits,
+                              const void* d_draft_logits, const int* d_draft_tokens, const float* d_uniforms,
+                              int* d_accept_len, int* d_out_offsets, int* d_out_tokens, float* d_draft_probs,
+                              void* stream) {
+  int st = check_spec_users(B, h_L, V);
+  if (st != DIPSD_OK) return st;
+  long long sum_l = 0, sum_t = 0;
+  for (int i = 0; i < B; ++i) {
+    sum_l += h_L[i];
+    sum_t += h_L[i] + 1;
+  }
+  if (sum_t > DIPSD_NOALLOC_MAX_POSITIONS) return DIPSD_ERR_UNSUPPORTED;
+  bool vec_ok = false;
+  st = check_spec_buffers(logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
+                          d_out_offsets, d_out_tokens, d_draft_probs, static_cast<int>(sum_l), V, &vec_ok);
+  if (st != DIPSD_OK) return st;
+  SpecPlan pl;
+  plan_spec(B, h_L, V, logit_dtype == DIPSD_BF16 ? 2 : 4, vec_ok, pl);
+  if (kStatusBytes + pl.ws_bytes > kNoAllocScratchBytes) return DIPSD_ERR_UNSUPPORTED;
+  uint8_t* ws = noalloc_scratch();
+  if (!ws) return DIPSD_ERR_CUDA;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(ws, 0, kStatusBytes, s) != cudaSuccess) return DIPSD_ERR_CUDA;
+  st = run_spec(pl, logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
+                d_out_offsets, d_out_tokens, d_draft_probs, reinterpret_cast<unsigned*>(ws), ws + kStatusBytes, s,
+                true);
   return st != DIPSD_OK ? st : cuda_status();
 }
 

@@ -31,8 +31,9 @@ EXPORTS = (
     "dipsd_status_string", "dipsd_abi_version", "dipsd_launch_count",
     "dipsd_verify_attention_workspace_size", "dipsd_verify_attention",
     "dipsd_spec_verify_workspace_size", "dipsd_spec_verify",
-    "dipsd_verify_batch_workspace_size", "dipsd_verify_batch",
+    "dipsd_verify_batch_workspace_size", "dipsd_verify_batch", "dipsd_spec_verify_noalloc",
 )
+NOALLOC_MAX_POSITIONS = 4096
 
 _lib: Optional[ctypes.CDLL] = None
 _i32p = ctypes.POINTER(ctypes.c_int)
@@ -74,6 +75,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.dipsd_verify_batch.argtypes = [_i, _i32p, _i, _i32p, _i32p, _vp, _vp, _vp, _i, _vp, _i, _i, _i, _i,
                                        ctypes.c_float, _vp, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
                                        _vp, _sz, _vp]
+    lib.dipsd_spec_verify_noalloc.restype = _i
+    lib.dipsd_spec_verify_noalloc.argtypes = [_i, _i32p, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]
     _lib = lib
     return lib
 
