@@ -12,6 +12,8 @@
 
 #include "dipsd.h"
 #include "attention.cuh"
+#include "attention_tc.cuh"
+#include "spec_generic.cuh"
 #include "spec_verify.cuh"
 
 namespace dipsd {
@@ -105,6 +107,18 @@ cudaError_t launch(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
   return e;
 }
 
+// Raises a kernel's dynamic shared memory limit once per device.
+template <typename K>
+bool allow_smem(K kernel, int bytes, bool* done) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
+  if (done[dev]) return true;
+  if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) != cudaSuccess)
+    return false;
+  done[dev] = true;
+  return true;
+}
+
 // =================================================================== attention
 struct AttnPlan {
   int B = 0, Hq = 0, Hkv = 0, G = 0, D = 0;
@@ -118,11 +132,6 @@ struct AttnPlan {
   size_t ws_bytes = 0;  // attention region only (excludes the status word)
 };
 
-int attn_stages(int D, int NW) { return D == 128 ? (NW == 4 ? 3 : 4) : 4; }
-
-size_t attn_smem(int D, int stages) {
-  return static_cast<size_t>(stages) * 2 * kAttnTile * D * 2 + 2 * stages * sizeof(uint64_t) + 1024;
-}
 
 // Validates the per-user attention arguments.
 int check_attn_users(int B, const int* L, const int* ctx, int Hq, int Hkv, int D) {
@@ -151,13 +160,12 @@ void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int
     max_m = std::max(max_m, pl.G * (L[i] + 1));
     max_tiles = std::max(max_tiles, (ctx[i] + L[i] + 1 + kAttnTile - 1) / kAttnTile);
   }
-  pl.NW = max_m <= 64 ? 4 : 8;
-  pl.stages = attn_stages(D, pl.NW);
-  pl.smem = attn_smem(D, pl.stages);
-  const int rows_cta = pl.NW * 16;
-  const int per_sm_smem = static_cast<int>((228 * 1024) / (pl.smem + 1024));
-  const int per_sm_regs = 65536 / ((pl.NW + 1) * 32 * 168);
-  const int slots = sms * std::max(1, std::min(per_sm_smem, per_sm_regs));
+  // tcgen05 kernel: 128 rows per CTA, one CTA per SM (its shared memory)
+  pl.NW = 8;
+  pl.stages = kTcStages;
+  pl.smem = D == 128 ? TcSmem<128>::kAlloc : TcSmem<64>::kAlloc;
+  const int rows_cta = 128;
+  const int slots = sms;
 
   int forced = 0;
   if (const char* e = std::getenv("DIPSD_ATTN_SPLIT_TILES")) forced = std::atoi(e);
@@ -181,7 +189,10 @@ void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int
       max_item = std::max(max_item, item);
     }
     if (items > (1ll << 30)) continue;
-    const double cost = total / slots + max_item;
+    // items are near-uniform (one split length): waves x longest item, but
+    // never better than perfect balance plus one item
+    const double waves = std::ceil(static_cast<double>(items) / slots);
+    const double cost = std::max(waves * max_item, total / slots + 0.5 * max_item);
     if (cost < best - 1e-9) { best = cost; best_c = c; }
     if (forced > 0) break;
   }
@@ -240,26 +251,17 @@ void fill_attn_params(AttnParams<CAP>& p, const AttnPlan& pl, const void* q, voi
   for (int i = 0; i < pl.B; ++i) { p.part_off[i] = pl.part_off[i]; p.u[i] = pl.u[i]; }
 }
 
-template <int D, int NW, int CAP>
-int launch_attention_t(const AttnPlan& pl, const AttnParams<CAP>& p, const CUtensorMap& tk,
-                       const CUtensorMap& tv, cudaStream_t s, bool pdl) {
-  constexpr int STAGES = (D == 128) ? (NW == 4 ? 3 : 4) : 4;
-  auto kern = verify_attention_kernel<D, NW, STAGES, CAP>;
+template <int D, int CAP>
+int launch_attention_tc_t(const AttnPlan& pl, const AttnParams<CAP>& p, const CUtensorMap& tk,
+                          const CUtensorMap& tv, cudaStream_t s, bool pdl) {
+  auto kern = verify_attention_tc_kernel<D, CAP>;
   static std::mutex mu;
   static bool attr_done[64] = {};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return DIPSD_ERR_CUDA;
   {
     std::lock_guard<std::mutex> lock(mu);
-    if (!attr_done[dev]) {
-      if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               static_cast<int>(attn_smem(D, STAGES))) != cudaSuccess)
-        return DIPSD_ERR_CUDA;
-      attr_done[dev] = true;
-    }
+    if (!allow_smem(kern, TcSmem<D>::kAlloc, attr_done)) return DIPSD_ERR_CUDA;
   }
-  if (launch(kern, dim3(pl.n_items), dim3((NW + 1) * 32), attn_smem(D, STAGES), s, 0, pdl, p, tk, tv) !=
-      cudaSuccess)
+  if (launch(kern, dim3(pl.n_items), dim3(kTcThreads), TcSmem<D>::kAlloc, s, 0, pdl, p, tk, tv) != cudaSuccess)
     return DIPSD_ERR_CUDA;
   if (pl.n_merge > 0) {
     auto mk = verify_attention_merge_kernel<D, CAP>;
@@ -279,11 +281,8 @@ int run_attention_cap(const AttnPlan& pl, const void* q, const void* kc, const v
   if (!encode_cache_map(&tk, kc, num_blocks, pl.Hkv, pl.D) ||
       !encode_cache_map(&tv, vc, num_blocks, pl.Hkv, pl.D))
     return DIPSD_ERR_CUDA;
-  if (pl.D == 128)
-    return pl.NW == 4 ? launch_attention_t<128, 4, CAP>(pl, p, tk, tv, s, pdl)
-                      : launch_attention_t<128, 8, CAP>(pl, p, tk, tv, s, pdl);
-  return pl.NW == 4 ? launch_attention_t<64, 4, CAP>(pl, p, tk, tv, s, pdl)
-                    : launch_attention_t<64, 8, CAP>(pl, p, tk, tv, s, pdl);
+  return pl.D == 128 ? launch_attention_tc_t<128, CAP>(pl, p, tk, tv, s, pdl)
+                     : launch_attention_tc_t<64, CAP>(pl, p, tk, tv, s, pdl);
 }
 
 int run_attention(const AttnPlan& pl, const void* q, const void* kc, const void* vc, int num_blocks,
@@ -312,10 +311,15 @@ int check_attn_buffers(const void* q, const void* kc, const void* vc, int num_bl
 // ===================================================================== spec
 struct SpecPlan {
   int B = 0, V = 0, vec = 1, nvec = 0, cl1 = 1, cl2 = 1;
+  bool staged = false;  // shared-memory staged kernels (16-byte aligned rows)
+  int slice_bytes = 0;  // staged: bytes of one row slice per CTA
   int sum_t = 0, sum_l = 0;
   std::vector<int> q_off, l_off;
   size_t ws_bytes = 0;  // spec region only
 };
+
+constexpr int kStagedSliceCap = 100 * 1024;  // per row; two rows per CTA
+constexpr int kStagedChunkVecs = kStagedWarps * 32 * kMaxGroups;  // slice limit from the group table
 
 int check_spec_users(int B, const int* L, int V) {
   if (B < 1 || B > kMaxUsers || !L || V < 1) return DIPSD_ERR_INVALID_ARG;
@@ -336,6 +340,18 @@ void plan_spec(int B, const int* L, int V, int elem, bool vec_ok, SpecPlan& pl) 
   pl.nvec = V / pl.vec;
   pl.cl1 = cluster_for(pl.nvec);
   pl.cl2 = cluster_for(pl.nvec);
+  pl.staged = false;
+  if (vec_ok) {
+    // staged path: a cluster of up to 8 CTAs per row, each holding one slice
+    int cl = pl.nvec >= kMaxCluster * 1024 ? kMaxCluster : std::max(1, (pl.nvec + 1023) / 1024);
+    while (cl < kMaxCluster && static_cast<long long>((pl.nvec + cl - 1) / cl) * 16 > kStagedSliceCap) ++cl;
+    const int slice_vecs = (pl.nvec + cl - 1) / cl;
+    if (static_cast<long long>(slice_vecs) * 16 <= kStagedSliceCap && slice_vecs <= kStagedChunkVecs) {
+      pl.staged = true;
+      pl.cl1 = pl.cl2 = cl;
+      pl.slice_bytes = slice_vecs * 16;
+    }
+  }
   pl.q_off.assign(B + 1, 0);
   pl.l_off.assign(B + 1, 0);
   for (int i = 0; i < B; ++i) {
@@ -344,16 +360,37 @@ void plan_spec(int B, const int* L, int V, int elem, bool vec_ok, SpecPlan& pl) 
   }
   pl.sum_t = pl.q_off[B];
   pl.sum_l = pl.l_off[B];
-  pl.ws_bytes = align_up(static_cast<size_t>(pl.sum_t) * sizeof(float4), 256) + align_up(pl.sum_t, 256);
+  pl.ws_bytes = align_up(static_cast<size_t>(pl.sum_t) * sizeof(SpecStat), 256) + align_up(pl.sum_t, 256);
 }
+
 
 template <typename T, int VEC, int CAP>
 int launch_spec_t(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s, bool pdl) {
-  if (launch(spec_stats_kernel<T, VEC, CAP>, dim3(pl.sum_t * pl.cl1), dim3(kSpecThreads), 0, s, pl.cl1, pdl,
-             p) != cudaSuccess)
+  if (launch(spec_stats_generic_kernel<T, VEC, CAP>, dim3(pl.sum_t * pl.cl1), dim3(kSpecThreads), 0, s, pl.cl1,
+             pdl, p) != cudaSuccess)
     return DIPSD_ERR_CUDA;
-  if (launch(spec_sample_kernel<T, VEC, CAP>, dim3(pl.B * pl.cl2), dim3(kSpecThreads), 0, s, pl.cl2, true,
-             p) != cudaSuccess)
+  if (launch(spec_sample_generic_kernel<T, VEC, CAP>, dim3(pl.B * pl.cl2), dim3(kSpecThreads), 0, s, pl.cl2,
+             true, p) != cudaSuccess)
+    return DIPSD_ERR_CUDA;
+  return DIPSD_OK;
+}
+
+template <typename T, int CAP>
+int launch_spec_staged_t(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s, bool pdl) {
+  static std::mutex mu;
+  static bool done1[64] = {}, done2[64] = {};
+  const int smem = 2 * pl.slice_bytes;
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    if (!allow_smem(spec_stats_kernel<T, CAP>, 2 * kStagedSliceCap, done1) ||
+        !allow_smem(spec_sample_kernel<T, CAP>, 2 * kStagedSliceCap, done2))
+      return DIPSD_ERR_CUDA;
+  }
+  if (launch(spec_stats_kernel<T, CAP>, dim3(pl.sum_t * pl.cl1), dim3(kStagedThreads), smem, s, pl.cl1, pdl, p,
+             pl.slice_bytes) != cudaSuccess)
+    return DIPSD_ERR_CUDA;
+  if (launch(spec_sample_kernel<T, CAP>, dim3(pl.B * pl.cl2), dim3(kStagedThreads), smem, s, pl.cl2, true, p,
+             pl.slice_bytes) != cudaSuccess)
     return DIPSD_ERR_CUDA;
   return DIPSD_OK;
 }
@@ -365,12 +402,15 @@ int run_spec_cap(const SpecPlan& pl, int dtype, const void* z, const void* w, co
   static thread_local SpecParams<CAP> p;
   std::memset(&p, 0, sizeof(p));
   p.z = z; p.w = w; p.draft_tokens = dt; p.uniforms = uni;
-  p.stats = reinterpret_cast<float4*>(region);
-  p.flags = region + align_up(static_cast<size_t>(pl.sum_t) * sizeof(float4), 256);
+  p.stats = region;
+  p.flags = region + align_up(static_cast<size_t>(pl.sum_t) * sizeof(SpecStat), 256);
   p.draft_probs = probs; p.accept_len = acc; p.out_offsets = offs; p.out_tokens = toks;
   p.status = status;
   p.B = pl.B; p.V = pl.V; p.nvec = pl.nvec;
   for (int i = 0; i <= pl.B; ++i) { p.q_off[i] = pl.q_off[i]; p.l_off[i] = pl.l_off[i]; }
+  if (pl.staged)
+    return dtype == DIPSD_BF16 ? launch_spec_staged_t<__nv_bfloat16, CAP>(pl, p, s, pdl)
+                               : launch_spec_staged_t<float, CAP>(pl, p, s, pdl);
   if (dtype == DIPSD_BF16)
     return pl.vec == 8 ? launch_spec_t<__nv_bfloat16, 8, CAP>(pl, p, s, pdl)
                        : launch_spec_t<__nv_bfloat16, 1, CAP>(pl, p, s, pdl);
@@ -410,7 +450,7 @@ int cuda_status() { return cudaGetLastError() == cudaSuccess ? DIPSD_OK : DIPSD_
 // statistics and acceptance bits for up to DIPSD_NOALLOC_MAX_POSITIONS
 // positions, laid out exactly like a dipsd_spec_verify workspace.
 constexpr size_t kNoAllocScratchBytes =
-    kStatusBytes + ((DIPSD_NOALLOC_MAX_POSITIONS * sizeof(float4) + 255) / 256) * 256 +
+    kStatusBytes + ((DIPSD_NOALLOC_MAX_POSITIONS * sizeof(SpecStat) + 255) / 256) * 256 +
     ((DIPSD_NOALLOC_MAX_POSITIONS + 255) / 256) * 256;
 
 }  // namespace

@@ -80,6 +80,10 @@ def check_spec(b, acc, offs, toks, probs, ref=None):
         np.testing.assert_allclose(pr[draft_pos, 0], ref["p_d"][draft_pos], atol=PROB_ATOL, rtol=0)
         np.testing.assert_allclose(pr[draft_pos, 1], ref["q_d"][draft_pos], atol=PROB_ATOL, rtol=0)
         assert np.all(pr[bonus_pos] == 0)
+        big = draft_pos[ref["p_d"][draft_pos] > 1e-6]
+        rel_p = float(np.max(np.abs(pr[big, 0] / ref["p_d"][big] - 1))) if big.size else 0.0
+    else:
+        rel_p = None
     near = oracle.decision_margins(ref, b.L, BAND)
     mismatch = np.zeros(B, dtype=bool)
     for i in range(B):
@@ -93,7 +97,7 @@ def check_spec(b, acc, offs, toks, probs, ref=None):
     assert far.size == 0, f"users {far.tolist()} differ from the oracle away from any decision boundary"
     n_mis = int(mismatch.sum())
     assert n_mis <= 1e-4 * positions, f"{n_mis} near-boundary mismatches out of {positions} positions"
-    return dict(users=B, positions=positions, near=int(near.sum()), mismatches=n_mis,
+    return dict(users=B, positions=positions, near=int(near.sum()), mismatches=n_mis, max_rel_err_p=rel_p,
                 emitted=int(offs[-1]), mean_accept=float(acc.mean()))
 
 
