@@ -156,6 +156,9 @@ __device__ __forceinline__ void dsmem_st_f32x4(uint32_t addr, float a, float b, 
                "f"(c), "f"(d)
                : "memory");
 }
+__device__ __forceinline__ void dsmem_st_f32x2(uint32_t addr, float a, float b) {
+  asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(addr), "f"(a), "f"(b) : "memory");
+}
 __device__ __forceinline__ void dsmem_st_f64(uint32_t addr, double a) {
   asm volatile("st.shared::cluster.f64 [%0], %1;" ::"r"(addr), "d"(a) : "memory");
 }

@@ -311,15 +311,13 @@ int check_attn_buffers(const void* q, const void* kc, const void* vc, int num_bl
 // ===================================================================== spec
 struct SpecPlan {
   int B = 0, V = 0, vec = 1, nvec = 0, cl1 = 1, cl2 = 1;
-  bool staged = false;  // shared-memory staged kernels (16-byte aligned rows)
-  int slice_bytes = 0;  // staged: bytes of one row slice per CTA
+  int nk = 0;  // register path: 16-byte vectors per thread per row (0 = generic path)
   int sum_t = 0, sum_l = 0;
   std::vector<int> q_off, l_off;
   size_t ws_bytes = 0;  // spec region only
 };
 
-constexpr int kStagedSliceCap = 100 * 1024;  // per row; two rows per CTA
-constexpr int kStagedChunkVecs = kStagedWarps * 32 * kMaxGroups;  // slice limit from the group table
+constexpr int kRegNk[] = {2, 4, 10, 20};
 
 int check_spec_users(int B, const int* L, int V) {
   if (B < 1 || B > kMaxUsers || !L || V < 1) return DIPSD_ERR_INVALID_ARG;
@@ -340,17 +338,15 @@ void plan_spec(int B, const int* L, int V, int elem, bool vec_ok, SpecPlan& pl) 
   pl.nvec = V / pl.vec;
   pl.cl1 = cluster_for(pl.nvec);
   pl.cl2 = cluster_for(pl.nvec);
-  pl.staged = false;
+  pl.nk = 0;
   if (vec_ok) {
-    // staged path: a cluster of up to 8 CTAs per row, each holding one slice
-    int cl = pl.nvec >= kMaxCluster * 1024 ? kMaxCluster : std::max(1, (pl.nvec + 1023) / 1024);
-    while (cl < kMaxCluster && static_cast<long long>((pl.nvec + cl - 1) / cl) * 16 > kStagedSliceCap) ++cl;
-    const int slice_vecs = (pl.nvec + cl - 1) / cl;
-    if (static_cast<long long>(slice_vecs) * 16 <= kStagedSliceCap && slice_vecs <= kStagedChunkVecs) {
-      pl.staged = true;
-      pl.cl1 = pl.cl2 = cl;
-      pl.slice_bytes = slice_vecs * 16;
-    }
+    // register path: a cluster of up to 8 CTAs per row, each thread holding
+    // nk vectors of its CTA's slice
+    const int cl = pl.nvec >= kMaxCluster * 1024 ? kMaxCluster : std::max(1, (pl.nvec + 1023) / 1024);
+    const int per_thread = ((pl.nvec + cl - 1) / cl + kRegThreads - 1) / kRegThreads;
+    for (int nk : kRegNk)
+      if (per_thread <= nk) { pl.nk = nk; break; }
+    if (pl.nk) pl.cl1 = pl.cl2 = cl;
   }
   pl.q_off.assign(B + 1, 0);
   pl.l_off.assign(B + 1, 0);
@@ -375,24 +371,25 @@ int launch_spec_t(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s, 
   return DIPSD_OK;
 }
 
-template <typename T, int CAP>
-int launch_spec_staged_t(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s, bool pdl) {
-  static std::mutex mu;
-  static bool done1[64] = {}, done2[64] = {};
-  const int smem = 2 * pl.slice_bytes;
-  {
-    std::lock_guard<std::mutex> lock(mu);
-    if (!allow_smem(spec_stats_kernel<T, CAP>, 2 * kStagedSliceCap, done1) ||
-        !allow_smem(spec_sample_kernel<T, CAP>, 2 * kStagedSliceCap, done2))
-      return DIPSD_ERR_CUDA;
-  }
-  if (launch(spec_stats_kernel<T, CAP>, dim3(pl.sum_t * pl.cl1), dim3(kStagedThreads), smem, s, pl.cl1, pdl, p,
-             pl.slice_bytes) != cudaSuccess)
+template <typename T, int NK, int CAP>
+int launch_spec_reg_t(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s, bool pdl) {
+  if (launch(spec_stats_kernel<T, NK, CAP>, dim3(pl.sum_t * pl.cl1), dim3(kRegThreads), 0, s, pl.cl1, pdl, p) !=
+      cudaSuccess)
     return DIPSD_ERR_CUDA;
-  if (launch(spec_sample_kernel<T, CAP>, dim3(pl.B * pl.cl2), dim3(kStagedThreads), smem, s, pl.cl2, true, p,
-             pl.slice_bytes) != cudaSuccess)
+  if (launch(spec_sample_kernel<T, NK, CAP>, dim3(pl.B * pl.cl2), dim3(kRegThreads), 0, s, pl.cl2, true, p) !=
+      cudaSuccess)
     return DIPSD_ERR_CUDA;
   return DIPSD_OK;
+}
+
+template <typename T, int CAP>
+int launch_spec_reg(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s, bool pdl) {
+  switch (pl.nk) {
+    case 2: return launch_spec_reg_t<T, 2, CAP>(pl, p, s, pdl);
+    case 4: return launch_spec_reg_t<T, 4, CAP>(pl, p, s, pdl);
+    case 10: return launch_spec_reg_t<T, 10, CAP>(pl, p, s, pdl);
+    default: return launch_spec_reg_t<T, 20, CAP>(pl, p, s, pdl);
+  }
 }
 
 template <int CAP>
@@ -408,9 +405,9 @@ int run_spec_cap(const SpecPlan& pl, int dtype, const void* z, const void* w, co
   p.status = status;
   p.B = pl.B; p.V = pl.V; p.nvec = pl.nvec;
   for (int i = 0; i <= pl.B; ++i) { p.q_off[i] = pl.q_off[i]; p.l_off[i] = pl.l_off[i]; }
-  if (pl.staged)
-    return dtype == DIPSD_BF16 ? launch_spec_staged_t<__nv_bfloat16, CAP>(pl, p, s, pdl)
-                               : launch_spec_staged_t<float, CAP>(pl, p, s, pdl);
+  if (pl.nk)
+    return dtype == DIPSD_BF16 ? launch_spec_reg<__nv_bfloat16, CAP>(pl, p, s, pdl)
+                               : launch_spec_reg<float, CAP>(pl, p, s, pdl);
   if (dtype == DIPSD_BF16)
     return pl.vec == 8 ? launch_spec_t<__nv_bfloat16, 8, CAP>(pl, p, s, pdl)
                        : launch_spec_t<__nv_bfloat16, 1, CAP>(pl, p, s, pdl);
