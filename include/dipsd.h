@@ -34,8 +34,10 @@
  *     matching *_workspace_size call returns for the same per-user arguments
  *     (on the same device).  Its first 16 bytes hold a device status word:
  *     kernels OR error bits into it (DIPSD_DEVERR_*) instead of trapping; zero
- *     it before a call whose status you want to read.  Calls that share a
- *     workspace must not overlap on the GPU.
+ *     it before a call whose status you want to read.  Zero the whole
+ *     workspace once before its first use (cudaMemset): the arrival counters
+ *     that follow the status word must start at zero, and every call leaves
+ *     them at zero.  Calls that share a workspace must not overlap on the GPU.
  */
 #ifndef DIPSD_H
 #define DIPSD_H
@@ -182,10 +184,11 @@ int dipsd_verify_batch(int B, const int* h_members, int M,
  * allocating library routine).
  *
  * Scratch lives in one static device array of the library, sized for at most
- * DIPSD_NOALLOC_MAX_POSITIONS verify positions (sum_i (L_i+1)); a larger batch
- * is rejected with DIPSD_ERR_UNSUPPORTED before anything is launched.  Every
- * GPU that loads the library holds that array (about 70 KB) until the process
- * exits.  The first call on a device looks up the array's device address with
+ * DIPSD_NOALLOC_MAX_POSITIONS verify positions (sum_i (L_i+1)) and 8 MiB in
+ * all (enough for bf16 logits with V up to about 160k at the maximum number of
+ * positions); a larger batch is rejected with DIPSD_ERR_UNSUPPORTED before
+ * anything is launched.  Every GPU that loads the library holds that 8 MiB
+ * array until the process exits.  The first call on a device looks up the array's device address with
  * that device current; make that first call before any stream capture.  All
  * calls share the one array: calls that overlap on the GPU (other streams,
  * other host threads) race and must be serialised by the caller.  Each call

@@ -20,6 +20,11 @@ namespace dipsd {
 namespace {
 
 constexpr size_t kStatusBytes = 256;
+// Arrival counters of the spec register path, at a fixed place right after
+// the status word whatever the entry point, so that every call finds them as
+// the last call left them (all zero).
+constexpr size_t kCounterBytes = (kCounterWords * sizeof(unsigned) + 255) / 256 * 256;
+constexpr size_t kHeaderBytes = kStatusBytes + kCounterBytes;
 constexpr int kCapSmall = 64;
 constexpr int kCapLarge = kMaxUsers;
 
@@ -311,13 +316,20 @@ int check_attn_buffers(const void* q, const void* kc, const void* vc, int num_bl
 // ===================================================================== spec
 struct SpecPlan {
   int B = 0, V = 0, vec = 1, nvec = 0, cl1 = 1, cl2 = 1;
-  int nk = 0;  // register path: 16-byte vectors per thread per row (0 = generic path)
+  int nk1 = 0, nk2 = 0;  // register path: vectors per lane and segment (0 = generic path)
+  int nseg1 = 0, nseg2 = 0, n_items1 = 0, n_items2 = 0;
   int sum_t = 0, sum_l = 0;
   std::vector<int> q_off, l_off;
+  size_t off_flags = 0, off_part1 = 0, off_part2 = 0;
   size_t ws_bytes = 0;  // spec region only
 };
 
-constexpr int kRegNk[] = {2, 4, 10, 20};
+// Register path segment sizes, largest first: a segment is 32 lanes x nk
+// 16-byte vectors of one row.
+constexpr int kNk1[] = {16, 8, 4};
+constexpr int kNk2[] = {8, 4, 2};
+// arrivals on one counter must fit its 16-bit count
+constexpr int kMaxArrivals = 60000;
 
 int check_spec_users(int B, const int* L, int V) {
   if (B < 1 || B > kMaxUsers || !L || V < 1) return DIPSD_ERR_INVALID_ARG;
@@ -332,22 +344,26 @@ int check_spec_users(int B, const int* L, int V) {
 
 int cluster_for(int nvec) { return std::max(1, std::min(kMaxCluster, (nvec + 2047) / 2048)); }
 
-void plan_spec(int B, const int* L, int V, int elem, bool vec_ok, SpecPlan& pl) {
+int ceil_div(int a, int b) { return (a + b - 1) / b; }
+
+// Largest segment size whose items still fill three quarters of the resident
+// warps (two 8-warp CTAs per SM); the smallest otherwise, or when sms <= 0
+// (the workspace bound, which must not depend on the device).
+template <size_t K>
+int pick_nk(const int (&opts)[K], long long rows, int nvec, int sms) {
+  if (sms <= 0) return opts[K - 1];
+  const long long want = static_cast<long long>(sms) * 16 * 3 / 4;
+  for (int nk : opts)
+    if (rows * ceil_div(nvec, 32 * nk) >= want) return nk;
+  return opts[K - 1];
+}
+
+void plan_spec(int B, const int* L, int V, int elem, bool vec_ok, int sms, SpecPlan& pl) {
   pl.B = B; pl.V = V;
   pl.vec = vec_ok ? 16 / elem : 1;
   pl.nvec = V / pl.vec;
   pl.cl1 = cluster_for(pl.nvec);
   pl.cl2 = cluster_for(pl.nvec);
-  pl.nk = 0;
-  if (vec_ok) {
-    // register path: a cluster of up to 8 CTAs per row, each thread holding
-    // nk vectors of its CTA's slice
-    const int cl = pl.nvec >= kMaxCluster * 1024 ? kMaxCluster : std::max(1, (pl.nvec + 1023) / 1024);
-    const int per_thread = ((pl.nvec + cl - 1) / cl + kRegThreads - 1) / kRegThreads;
-    for (int nk : kRegNk)
-      if (per_thread <= nk) { pl.nk = nk; break; }
-    if (pl.nk) pl.cl1 = pl.cl2 = cl;
-  }
   pl.q_off.assign(B + 1, 0);
   pl.l_off.assign(B + 1, 0);
   for (int i = 0; i < B; ++i) {
@@ -356,9 +372,47 @@ void plan_spec(int B, const int* L, int V, int elem, bool vec_ok, SpecPlan& pl) 
   }
   pl.sum_t = pl.q_off[B];
   pl.sum_l = pl.l_off[B];
-  pl.ws_bytes = align_up(static_cast<size_t>(pl.sum_t) * sizeof(SpecStat), 256) + align_up(pl.sum_t, 256);
+  pl.nk1 = pl.nk2 = 0;
+  pl.nseg1 = pl.nseg2 = pl.n_items1 = pl.n_items2 = 0;
+  size_t o = align_up(static_cast<size_t>(pl.sum_t) * sizeof(SpecStat), 256);
+  pl.off_flags = o;
+  o += align_up(pl.sum_t, 256);
+  pl.off_part1 = pl.off_part2 = o;
+  if (vec_ok) {
+    const int nk1 = pick_nk(kNk1, pl.sum_t + pl.sum_l, pl.nvec, sms);
+    const int nk2 = pick_nk(kNk2, B, pl.nvec, sms);
+    const int nseg1 = ceil_div(pl.nvec, 32 * nk1), nseg2 = ceil_div(pl.nvec, 32 * nk2);
+    const long long items1 = static_cast<long long>(pl.sum_t + pl.sum_l) * nseg1;
+    const long long items2 = static_cast<long long>(B) * nseg2;
+    if (2 * nseg1 <= kMaxArrivals && nseg2 <= kMaxArrivals && items1 < (1ll << 31) && items2 < (1ll << 31)) {
+      pl.nk1 = nk1; pl.nk2 = nk2;
+      pl.nseg1 = nseg1; pl.nseg2 = nseg2;
+      pl.n_items1 = static_cast<int>(items1);
+      pl.n_items2 = static_cast<int>(items2);
+      o += align_up(static_cast<size_t>(items1) * sizeof(float4), 256);
+      pl.off_part2 = o;
+      o += align_up(static_cast<size_t>(items2) * sizeof(float4), 256);
+    }
+  }
+  pl.ws_bytes = o;
 }
 
+// Spec workspace that covers every plan a call with these sizes can get
+// (either logit type, aligned or not, any device): the smallest segments.
+size_t spec_ws_need(int B, const int* L, int V) {
+  SpecPlan pl;
+  plan_spec(B, L, V, 2, false, 0, pl);
+  size_t need = pl.ws_bytes;
+  if (V % 8 == 0) {
+    plan_spec(B, L, V, 2, true, 0, pl);
+    need = std::max(need, pl.ws_bytes);
+  }
+  if (V % 4 == 0) {
+    plan_spec(B, L, V, 4, true, 0, pl);
+    need = std::max(need, pl.ws_bytes);
+  }
+  return need;
+}
 
 template <typename T, int VEC, int CAP>
 int launch_spec_t(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s, bool pdl) {
@@ -371,24 +425,30 @@ int launch_spec_t(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s, 
   return DIPSD_OK;
 }
 
-template <typename T, int NK, int CAP>
+template <typename T, int NK2, int CAP>
+int launch_spec_sample_t(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s) {
+  return launch(spec_sample_kernel<T, NK2, CAP>, dim3(ceil_div(pl.n_items2, kRegWarps)), dim3(kRegThreads), 0, s,
+                1, true, p) == cudaSuccess ? DIPSD_OK : DIPSD_ERR_CUDA;
+}
+
+template <typename T, int NK1, int CAP>
 int launch_spec_reg_t(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s, bool pdl) {
-  if (launch(spec_stats_kernel<T, NK, CAP>, dim3(pl.sum_t * pl.cl1), dim3(kRegThreads), 0, s, pl.cl1, pdl, p) !=
-      cudaSuccess)
+  if (launch(spec_stats_kernel<T, NK1, CAP>, dim3(ceil_div(pl.n_items1, kRegWarps)), dim3(kRegThreads), 0, s, 1,
+             pdl, p) != cudaSuccess)
     return DIPSD_ERR_CUDA;
-  if (launch(spec_sample_kernel<T, NK, CAP>, dim3(pl.B * pl.cl2), dim3(kRegThreads), 0, s, pl.cl2, true, p) !=
-      cudaSuccess)
-    return DIPSD_ERR_CUDA;
-  return DIPSD_OK;
+  switch (pl.nk2) {
+    case 8: return launch_spec_sample_t<T, 8, CAP>(pl, p, s);
+    case 4: return launch_spec_sample_t<T, 4, CAP>(pl, p, s);
+    default: return launch_spec_sample_t<T, 2, CAP>(pl, p, s);
+  }
 }
 
 template <typename T, int CAP>
 int launch_spec_reg(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s, bool pdl) {
-  switch (pl.nk) {
-    case 2: return launch_spec_reg_t<T, 2, CAP>(pl, p, s, pdl);
-    case 4: return launch_spec_reg_t<T, 4, CAP>(pl, p, s, pdl);
-    case 10: return launch_spec_reg_t<T, 10, CAP>(pl, p, s, pdl);
-    default: return launch_spec_reg_t<T, 20, CAP>(pl, p, s, pdl);
+  switch (pl.nk1) {
+    case 16: return launch_spec_reg_t<T, 16, CAP>(pl, p, s, pdl);
+    case 8: return launch_spec_reg_t<T, 8, CAP>(pl, p, s, pdl);
+    default: return launch_spec_reg_t<T, 4, CAP>(pl, p, s, pdl);
   }
 }
 
@@ -400,12 +460,18 @@ int run_spec_cap(const SpecPlan& pl, int dtype, const void* z, const void* w, co
   std::memset(&p, 0, sizeof(p));
   p.z = z; p.w = w; p.draft_tokens = dt; p.uniforms = uni;
   p.stats = region;
-  p.flags = region + align_up(static_cast<size_t>(pl.sum_t) * sizeof(SpecStat), 256);
+  p.flags = region + pl.off_flags;
+  p.part1 = reinterpret_cast<float4*>(region + pl.off_part1);
+  p.part2 = reinterpret_cast<float4*>(region + pl.off_part2);
+  p.counters = reinterpret_cast<unsigned*>(reinterpret_cast<uint8_t*>(status) + kStatusBytes);
+  p.sum_t = pl.sum_t;
+  p.nseg1 = pl.nseg1; p.nseg2 = pl.nseg2;
+  p.n_items1 = pl.n_items1; p.n_items2 = pl.n_items2;
   p.draft_probs = probs; p.accept_len = acc; p.out_offsets = offs; p.out_tokens = toks;
   p.status = status;
   p.B = pl.B; p.V = pl.V; p.nvec = pl.nvec;
   for (int i = 0; i <= pl.B; ++i) { p.q_off[i] = pl.q_off[i]; p.l_off[i] = pl.l_off[i]; }
-  if (pl.nk)
+  if (pl.nk1)
     return dtype == DIPSD_BF16 ? launch_spec_reg<__nv_bfloat16, CAP>(pl, p, s, pdl)
                                : launch_spec_reg<float, CAP>(pl, p, s, pdl);
   if (dtype == DIPSD_BF16)
@@ -443,12 +509,11 @@ int check_workspace(const void* ws, size_t have, size_t need) {
 int cuda_status() { return cudaGetLastError() == cudaSuccess ? DIPSD_OK : DIPSD_ERR_CUDA; }
 
 // ------------------------------------------------------- no-alloc scratch
-// Scratch of dipsd_spec_verify_noalloc: status word, per-position row
-// statistics and acceptance bits for up to DIPSD_NOALLOC_MAX_POSITIONS
-// positions, laid out exactly like a dipsd_spec_verify workspace.
-constexpr size_t kNoAllocScratchBytes =
-    kStatusBytes + ((DIPSD_NOALLOC_MAX_POSITIONS * sizeof(SpecStat) + 255) / 256) * 256 +
-    ((DIPSD_NOALLOC_MAX_POSITIONS + 255) / 256) * 256;
+// Scratch of dipsd_spec_verify_noalloc: the status word followed by a
+// dipsd_spec_verify workspace region (row statistics, acceptance bits,
+// segment partial sums and arrival counters).  8 MiB covers bf16 logits with
+// V up to about 160k at DIPSD_NOALLOC_MAX_POSITIONS positions.
+constexpr size_t kNoAllocScratchBytes = size_t(8) << 20;
 
 }  // namespace
 }  // namespace dipsd
@@ -496,7 +561,7 @@ size_t dipsd_verify_attention_workspace_size(int B, const int* h_L, const int* h
   if (!device_facts(f)) return 0;
   AttnPlan pl;
   plan_attention(B, h_L, h_ctx, nullptr, Hq, Hkv, D, f.sms, pl);
-  return kStatusBytes + pl.ws_bytes;
+  return kHeaderBytes + pl.ws_bytes;
 }
 
 int dipsd_verify_attention(int B, const int* h_L, const int* h_ctx, const void* d_q, const void* d_k_cache,
@@ -512,19 +577,17 @@ int dipsd_verify_attention(int B, const int* h_L, const int* h_ctx, const void* 
   if (!device_facts(f)) return DIPSD_ERR_CUDA;
   AttnPlan pl;
   plan_attention(B, h_L, h_ctx, nullptr, Hq, Hkv, D, f.sms, pl);
-  st = check_workspace(d_workspace, workspace_bytes, kStatusBytes + pl.ws_bytes);
+  st = check_workspace(d_workspace, workspace_bytes, kHeaderBytes + pl.ws_bytes);
   if (st != DIPSD_OK) return st;
   uint8_t* ws = static_cast<uint8_t*>(d_workspace);
   st = run_attention(pl, d_q, d_k_cache, d_v_cache, num_blocks, d_block_table, max_blocks, softmax_scale, d_out,
-                     reinterpret_cast<unsigned*>(ws), ws + kStatusBytes, static_cast<cudaStream_t>(stream), true);
+                     reinterpret_cast<unsigned*>(ws), ws + kHeaderBytes, static_cast<cudaStream_t>(stream), true);
   return st != DIPSD_OK ? st : cuda_status();
 }
 
 size_t dipsd_spec_verify_workspace_size(int B, const int* h_L, int V) {
   if (check_spec_users(B, h_L, V) != DIPSD_OK) return 0;
-  SpecPlan pl;
-  plan_spec(B, h_L, V, 2, false, pl);
-  return kStatusBytes + pl.ws_bytes;
+  return kHeaderBytes + spec_ws_need(B, h_L, V);
 }
 
 int dipsd_spec_verify(int B, const int* h_L, int V, int logit_dtype, const void* d_target_logits,
@@ -539,13 +602,15 @@ int dipsd_spec_verify(int B, const int* h_L, int V, int logit_dtype, const void*
   st = check_spec_buffers(logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
                           d_out_offsets, d_out_tokens, d_draft_probs, static_cast<int>(sum_l), V, &vec_ok);
   if (st != DIPSD_OK) return st;
-  SpecPlan pl;
-  plan_spec(B, h_L, V, logit_dtype == DIPSD_BF16 ? 2 : 4, vec_ok, pl);
-  st = check_workspace(d_workspace, workspace_bytes, kStatusBytes + pl.ws_bytes);
+  st = check_workspace(d_workspace, workspace_bytes, kHeaderBytes + spec_ws_need(B, h_L, V));
   if (st != DIPSD_OK) return st;
+  DeviceFacts f;
+  if (!device_facts(f)) return DIPSD_ERR_CUDA;
+  SpecPlan pl;
+  plan_spec(B, h_L, V, logit_dtype == DIPSD_BF16 ? 2 : 4, vec_ok, f.sms, pl);
   uint8_t* ws = static_cast<uint8_t*>(d_workspace);
   st = run_spec(pl, logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
-                d_out_offsets, d_out_tokens, d_draft_probs, reinterpret_cast<unsigned*>(ws), ws + kStatusBytes,
+                d_out_offsets, d_out_tokens, d_draft_probs, reinterpret_cast<unsigned*>(ws), ws + kHeaderBytes,
                 static_cast<cudaStream_t>(stream), true);
   return st != DIPSD_OK ? st : cuda_status();
 }
@@ -566,15 +631,17 @@ int dipsd_spec_verify_noalloc(int B, const int* h_L, int V, int logit_dtype, con
   st = check_spec_buffers(logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
                           d_out_offsets, d_out_tokens, d_draft_probs, static_cast<int>(sum_l), V, &vec_ok);
   if (st != DIPSD_OK) return st;
+  DeviceFacts f;
+  if (!device_facts(f)) return DIPSD_ERR_CUDA;
   SpecPlan pl;
-  plan_spec(B, h_L, V, logit_dtype == DIPSD_BF16 ? 2 : 4, vec_ok, pl);
-  if (kStatusBytes + pl.ws_bytes > kNoAllocScratchBytes) return DIPSD_ERR_UNSUPPORTED;
+  plan_spec(B, h_L, V, logit_dtype == DIPSD_BF16 ? 2 : 4, vec_ok, f.sms, pl);
+  if (kHeaderBytes + pl.ws_bytes > kNoAllocScratchBytes) return DIPSD_ERR_UNSUPPORTED;
   uint8_t* ws = noalloc_scratch();
   if (!ws) return DIPSD_ERR_CUDA;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (cudaMemsetAsync(ws, 0, kStatusBytes, s) != cudaSuccess) return DIPSD_ERR_CUDA;
   st = run_spec(pl, logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
-                d_out_offsets, d_out_tokens, d_draft_probs, reinterpret_cast<unsigned*>(ws), ws + kStatusBytes, s,
+                d_out_offsets, d_out_tokens, d_draft_probs, reinterpret_cast<unsigned*>(ws), ws + kHeaderBytes, s,
                 true);
   return st != DIPSD_OK ? st : cuda_status();
 }
@@ -605,9 +672,7 @@ size_t dipsd_verify_batch_workspace_size(int B, const int* h_members, int M, con
   if (!device_facts(f)) return 0;
   AttnPlan ap;
   plan_attention(B, L.data(), ctx.data(), h_members, Hq, Hkv, D, f.sms, ap);
-  SpecPlan sp;
-  plan_spec(B, L.data(), V, 2, false, sp);
-  return kStatusBytes + align_up(ap.ws_bytes, 256) + sp.ws_bytes;
+  return kHeaderBytes + align_up(ap.ws_bytes, 256) + spec_ws_need(B, L.data(), V);
 }
 
 int dipsd_verify_batch(int B, const int* h_members, int M, const int* h_L_all, const int* h_ctx_all,
@@ -638,18 +703,18 @@ int dipsd_verify_batch(int B, const int* h_members, int M, const int* h_L_all, c
   AttnPlan ap;
   plan_attention(B, L.data(), ctx.data(), h_members, Hq, Hkv, D, f.sms, ap);
   SpecPlan sp;
-  plan_spec(B, L.data(), V, logit_dtype == DIPSD_BF16 ? 2 : 4, vec_ok, sp);
+  plan_spec(B, L.data(), V, logit_dtype == DIPSD_BF16 ? 2 : 4, vec_ok, f.sms, sp);
   const size_t attn_region = align_up(ap.ws_bytes, 256);
-  st = check_workspace(d_workspace, workspace_bytes, kStatusBytes + attn_region + sp.ws_bytes);
+  st = check_workspace(d_workspace, workspace_bytes, kHeaderBytes + attn_region + sp.ws_bytes);
   if (st != DIPSD_OK) return st;
   uint8_t* ws = static_cast<uint8_t*>(d_workspace);
   unsigned* status = reinterpret_cast<unsigned*>(ws);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   st = run_attention(ap, d_q, d_k_cache, d_v_cache, num_blocks, d_block_table_all, max_blocks, softmax_scale,
-                     d_attn_out, status, ws + kStatusBytes, s, true);
+                     d_attn_out, status, ws + kHeaderBytes, s, true);
   if (st != DIPSD_OK) return st;
   st = run_spec(sp, logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
-                d_out_offsets, d_out_tokens, d_draft_probs, status, ws + kStatusBytes + attn_region, s, true);
+                d_out_offsets, d_out_tokens, d_draft_probs, status, ws + kHeaderBytes + attn_region, s, true);
   return st != DIPSD_OK ? st : cuda_status();
 }
 

@@ -11,6 +11,13 @@ constexpr int kSpecThreads = 256;
 constexpr int kSpecWarps = kSpecThreads / 32;
 constexpr int kMaxCluster = 8;
 constexpr unsigned kDevErrBadToken = 2u;
+// Arrival counters of the register path, in 32-bit words: one per verify
+// position; then one 64-bit word per user for the decisions (arrivals in the
+// high half, acceptance bit t of position t in the low half); then one per
+// user for the sampling segments.
+constexpr int kCntUser1 = kMaxUsers * (kMaxDraft + 1);
+constexpr int kCntUser2 = kCntUser1 + 2 * kMaxUsers;
+constexpr int kCounterWords = kCntUser2 + kMaxUsers;
 
 template <int CAP>
 struct SpecParams {
@@ -25,6 +32,11 @@ struct SpecParams {
   int* out_offsets;           // [B+1]
   int* out_tokens;            // [sum T]
   unsigned* status;
+  // register path only: segment partial sums and arrival counters
+  float4* part1;       // [n_items1] one per segment of every row
+  float4* part2;       // [n_items2] one per segment of the sampled rows
+  unsigned* counters;  // [kCounterWords], zero between calls
+  int sum_t, nseg1, nseg2, n_items1, n_items2;
   int B, V, nvec;             // nvec = V / VEC
   int q_off[CAP + 1];         // first verify position of user i
   int l_off[CAP + 1];         // first draft row of user i

@@ -3,27 +3,30 @@
 // rejection, emit one more token from the residual or, at the bonus position,
 // from the target distribution).  Register path for 16-byte aligned rows.
 //
-// Rows are read once, with every 16-byte load of a thread issued up front and
-// kept in registers (a slice of 256 threads x up to NK vectors per row), so a
-// CTA has its whole slice in flight at once; no shared-memory staging.
+// Both kernels are flat over warps.  A work item is one warp-sized segment of
+// one row: 32 lanes x NK 16-byte vectors, lane-interleaved so that every load
+// instruction of the warp reads 512 contiguous bytes, all of a lane's loads
+// issued before the first use.  Items spread evenly over the SMs whatever the
+// mix of draft lengths.  Segments meet through arrival counters in global
+// memory: the warp that delivers the last segment of a position (or of a
+// user) goes on with the step that needs them all, and no warp ever waits for
+// another.
 //
-// Pass 1 (spec_stats_kernel) -- one thread-block cluster per verify position.
-// Each CTA owns a slice of the target-logit row (and of the draft-logit row at
-// draft positions).  A thread takes its maximum m, picks the integer reference
-// c = ceil(m log2 e) and sums 2^(x log2 e - c) (two FFMA and one ex2 per
-// logit).  Because references are integers, every rescale between threads,
-// warps, CTAs and cluster ranks is an exact power of two; partial sums combine
-// as float-float pairs and the row normaliser is kept in fp64.  Rank 0 forms
-// p_t(d), q_t(d) and takes the acceptance decision u_acc * q_t(d) < p_t(d).
+// spec_stats_kernel: items are the segments of every target row z_t and every
+// draft row w_t.  A warp takes the integer reference c = ceil(m log2 e) of its
+// segment maximum m and sums 2^(x log2 e - c) (two FFMA and one ex2 per
+// logit).  References are integers, so partial sums combine by exact
+// power-of-two rescaling as float-float pairs.  The last segment of position
+// t combines the row sums, forms p_t(d), q_t(d) and decides
+// u_acc * q_t(d) < p_t(d); the last decided position of user i counts the
+// leading accepts a_i.
 //
-// Pass 2 (spec_sample_kernel) -- one cluster per user.  Warp ballots over the
-// acceptance bits give a_i and the packed output offset.  The slices of the
-// rows at position a_i are loaded the same way; weights (max(0, p - q) up to a
-// common factor, or p at the bonus position) use the pass-1 exponential.  Each
-// warp covers 32 consecutive vectors (256 tokens) per step -- a group -- and
-// keeps every group total; slice totals are exchanged through distributed
-// shared memory, and the CTA holding u * total descends slice -> group ->
-// lane -> token on the very same fp32 partial sums, so the descent always
+// spec_sample_kernel: items are the segments of the rows at position a_i of
+// every user.  A warp computes the sampling weights (max(0, p - q) up to a
+// common factor, or p at the bonus position) and stores its segment's total,
+// summed in token order: fp32 scans over 32-vector groups, float-float across
+// groups.  The last segment of user i locates u * total: segment, group, lane
+// and token, replaying the very sums that produced the totals, so the descent
 // lands in the cell the totals point to.
 #pragma once
 
@@ -35,26 +38,29 @@ constexpr float kLog2e = 1.4426950408889634f;
 // log2(e) = kLog2eHi + kLog2eLo (the fp32 rounding and its remainder).
 constexpr float kLog2eHi = 1.44269502162933349609375f;
 constexpr float kLog2eLo = 1.925963033500651e-8f;
-// ln 2 = kLn2Hi + kLn2Lo; kLn2Hi has 16 significant bits, so c * kLn2Hi is
-// exact for integers |c| < 2^8 (Cody and Waite's argument reduction).
-constexpr float kLn2Hi = 0.693145751953125f;
-constexpr float kLn2Lo = 1.42860682030941723212e-6f;
 constexpr int kEmptyRef = -(1 << 29);
 constexpr int kRegThreads = 256;
 constexpr int kRegWarps = kRegThreads / 32;
 
 // Row statistics of one verify position, relative to integer references:
-// sz = sum_v 2^(z_v log2 e - cz), sw likewise for the draft row.
+// sz = sum_v 2^(z_v log2 e - cz), sw likewise for the draft row; sz / sw, the
+// scale of q against p in the residual, split into two floats.
 struct SpecStat {
   double sz, sw;
   int cz, cw;
-  int pad0, pad1;
+  float khi, klo;
+};
+// The part of SpecStat the sampling weights need (its second 16 bytes).
+struct WRef {
+  int cz, cw;
+  float khi, klo;
 };
 
 // --------------------------------------------------------- float-float sums
 struct FF {
   float hi, lo;
 };
+// Commutative bit for bit: the TwoSum error term is exact.
 __device__ __forceinline__ FF ff_add(FF a, FF b) {
   const float s = __fadd_rn(a.hi, b.hi);
   const float bb = __fsub_rn(s, a.hi);
@@ -63,7 +69,15 @@ __device__ __forceinline__ FF ff_add(FF a, FF b) {
   const float hi = __fadd_rn(s, lo);
   return FF{hi, __fsub_rn(lo, __fsub_rn(hi, s))};
 }
-__device__ __forceinline__ FF ff_scale(FF a, int k) { return FF{scalbnf(a.hi, k), scalbnf(a.lo, k)}; }
+// 2^k for k <= 0 as an exact float (0 below the normal range).
+__device__ __forceinline__ float pow2_nonpos(int k) {
+  return k < -126 ? 0.f : __int_as_float((k + 127) << 23);
+}
+// a * 2^k for k <= 0 (exact for normal results)
+__device__ __forceinline__ FF ff_scale(FF a, int k) {
+  const float f = pow2_nonpos(k);
+  return FF{__fmul_rn(a.hi, f), __fmul_rn(a.lo, f)};
+}
 __device__ __forceinline__ FF ff_neg(FF a) { return FF{-a.hi, -a.lo}; }
 __device__ __forceinline__ FF ff_sub(FF a, FF b) { return ff_add(a, ff_neg(b)); }
 // a > b for float-float values
@@ -77,6 +91,9 @@ __device__ __forceinline__ FF ff_mul_f(FF a, float u) {
   const float e = __fmaf_rn(a.hi, u, -p);
   return ff_add(FF{p, 0.f}, FF{e, __fmul_rn(a.lo, u)});
 }
+__device__ __forceinline__ FF ff_shfl(FF v, int src) {
+  return FF{__shfl_sync(0xffffffffu, v.hi, src), __shfl_sync(0xffffffffu, v.lo, src)};
+}
 // inclusive warp scan of float-float values
 __device__ __forceinline__ FF warp_ff_scan(FF v, int lane) {
 #pragma unroll
@@ -85,6 +102,24 @@ __device__ __forceinline__ FF warp_ff_scan(FF v, int lane) {
     y.hi = __shfl_up_sync(0xffffffffu, v.hi, o);
     y.lo = __shfl_up_sync(0xffffffffu, v.lo, o);
     if (lane >= o) v = ff_add(y, v);
+  }
+  return v;
+}
+// the scan value of the previous lane (0 at lane 0)
+__device__ __forceinline__ FF warp_ff_exclusive(FF incl, int lane) {
+  FF e;
+  e.hi = __shfl_up_sync(0xffffffffu, incl.hi, 1);
+  e.lo = __shfl_up_sync(0xffffffffu, incl.lo, 1);
+  return lane == 0 ? FF{0.f, 0.f} : e;
+}
+// warp total of float-float values (every lane gets the same bits)
+__device__ __forceinline__ FF warp_ff_sum(FF v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    FF y;
+    y.hi = __shfl_xor_sync(0xffffffffu, v.hi, o);
+    y.lo = __shfl_xor_sync(0xffffffffu, v.lo, o);
+    v = ff_add(v, y);
   }
   return v;
 }
@@ -126,7 +161,18 @@ __device__ __forceinline__ float ex2_ref(float x, float cf) {
 }
 __device__ __forceinline__ float ex2_ref(float x, int c) { return ex2_ref(x, static_cast<float>(c)); }
 
-// ------------------------------------------------------ register slices
+// ------------------------------------------------------ arrival counters
+// Counters are zero between calls: the last arrival of a call stores 0.
+// Returns the arrival number (1-based).  The add is a release of the calling
+// thread's earlier writes and an acquire of those of earlier arrivals; the
+// arriving lane passes them on to its warp with __syncwarp.
+__device__ __forceinline__ unsigned counter_arrive(unsigned* ctr) {
+  unsigned old;
+  asm volatile("atom.add.acq_rel.gpu.u32 %0, [%1], 1;" : "=r"(old) : "l"(ctr) : "memory");
+  return old + 1u;
+}
+
+// ------------------------------------------------------ register segments
 template <typename T>
 struct Vec16;
 template <>
@@ -150,166 +196,122 @@ struct Vec16<float> {
   }
 };
 
-// Largest element of one 16-byte vector (bf16 pairs compared packed).
-template <typename T>
-__device__ __forceinline__ float vec_max(const uint4& r) {
-  if constexpr (sizeof(T) == 2) {
-    uint32_t a, b, c;
-    asm("max.bf16x2 %0, %1, %2;" : "=r"(a) : "r"(r.x), "r"(r.y));
-    asm("max.bf16x2 %0, %1, %2;" : "=r"(b) : "r"(r.z), "r"(r.w));
-    asm("max.bf16x2 %0, %1, %2;" : "=r"(c) : "r"(a), "r"(b));
-    return fmaxf(__uint_as_float(c << 16), __uint_as_float(c & 0xFFFF0000u));
-  } else {
-    return fmaxf(fmaxf(__uint_as_float(r.x), __uint_as_float(r.y)), fmaxf(__uint_as_float(r.z), __uint_as_float(r.w)));
-  }
+// A lane's vectors in the segment that starts at vector vb:
+// vb + k * 32 + lane < nvec for k < the returned count (at most nk).
+__device__ __forceinline__ int lane_vectors(int nvec, int vb, int lane, int nk) {
+  const int n = nvec - vb - lane;
+  return n > 0 ? min(nk, (n + 31) >> 5) : 0;
 }
 
-// Slice of CTA `rank` in units of 16-byte vectors.
-__device__ __forceinline__ void slice_bounds(int nvec, uint32_t rank, uint32_t csize, int& sb, int& se) {
-  sb = static_cast<int>((static_cast<long long>(rank) * nvec) / csize);
-  se = static_cast<int>((static_cast<long long>(rank + 1) * nvec) / csize);
-}
-
-// Loads this thread's vectors of a slice: vector sb + k*kRegThreads + tid.
+// Loads a lane's nv vectors of a segment (the rest of r is zeroed).
 template <int NK>
-__device__ __forceinline__ void load_slice(const uint8_t* row, int sb, int se, int tid, uint4 (&r)[NK]) {
+__device__ __forceinline__ void load_segment(const void* row, int vb, int lane, int nv, uint4 (&r)[NK]) {
+  const uint8_t* q = static_cast<const uint8_t*>(row) + (static_cast<size_t>(vb) + lane) * 16;
 #pragma unroll
-  for (int k = 0; k < NK; ++k) {
-    const int v = sb + k * kRegThreads + tid;
-    r[k] = v < se ? ldg_stream_v4(row + static_cast<size_t>(v) * 16) : make_uint4(0, 0, 0, 0);
-  }
+  for (int k = 0; k < NK; ++k)
+    r[k] = k < nv ? ldg_stream_v4(q + static_cast<size_t>(k) * 512) : make_uint4(0u, 0u, 0u, 0u);
 }
 
-// Thread partial sum of 2^(x log2 e - c) over its loaded vectors.
-template <typename T, int NK>
-__device__ __forceinline__ RefSum thread_refsum(const uint4 (&r)[NK], int sb, int se, int tid) {
-  constexpr int N = Vec16<T>::N;
-  float m = -INFINITY;
+// Largest logit among a lane's vectors k0 <= k < k0 + KG, k < nv (bf16 pairs
+// compared packed).
+template <typename T, int NK, int KG>
+__device__ __forceinline__ float lane_max(const uint4 (&r)[NK], int k0, int nv) {
+  if constexpr (sizeof(T) == 2) {
+    uint32_t pm = 0xFF80FF80u;  // packed -inf, -inf
 #pragma unroll
-  for (int k = 0; k < NK; ++k) {
-    if (sb + k * kRegThreads + tid < se) m = fmaxf(m, vec_max<T>(r[k]));
-  }
-  if (!(m > -INFINITY)) return RefSum{kEmptyRef, FF{0.f, 0.f}};
-  const float cf = fminf(fmaxf(ceilf(m * kLog2e), -1048576.f), 1048576.f);
-  KahanSum acc;
-#pragma unroll
-  for (int k = 0; k < NK; ++k) {
-    if (sb + k * kRegThreads + tid < se) {
-      float x[N];
-      Vec16<T>::unpack(r[k], x);
-      float e[N];
-#pragma unroll
-      for (int q = 0; q < N; ++q) e[q] = ex2_ref(x[q], cf);
-      float sv;
-      if constexpr (N == 8) {
-        sv = ((e[0] + e[1]) + (e[2] + e[3])) + ((e[4] + e[5]) + (e[6] + e[7]));
-      } else {
-        sv = (e[0] + e[1]) + (e[2] + e[3]);
+    for (int k = k0; k < k0 + KG; ++k) {
+      if (k < nv) {
+        uint32_t a, b;
+        asm("max.bf16x2 %0, %1, %2;" : "=r"(a) : "r"(r[k].x), "r"(r[k].y));
+        asm("max.bf16x2 %0, %1, %2;" : "=r"(b) : "r"(r[k].z), "r"(r[k].w));
+        asm("max.bf16x2 %0, %1, %2;" : "=r"(a) : "r"(a), "r"(b));
+        asm("max.bf16x2 %0, %1, %2;" : "=r"(pm) : "r"(pm), "r"(a));
       }
-      acc.add(sv);
     }
+    return fmaxf(__uint_as_float(pm << 16), __uint_as_float(pm & 0xFFFF0000u));
+  } else {
+    float m = -INFINITY;
+#pragma unroll
+    for (int k = k0; k < k0 + KG; ++k)
+      if (k < nv)
+        m = fmaxf(m, fmaxf(fmaxf(__uint_as_float(r[k].x), __uint_as_float(r[k].y)),
+                           fmaxf(__uint_as_float(r[k].z), __uint_as_float(r[k].w))));
+    return m;
   }
-  return RefSum{static_cast<int>(cf), FF{acc.s, -acc.c}};
 }
 
-// ------------------------------------------------------------------ pass 1
-template <typename T, int NK, int CAP>
-__global__ void __launch_bounds__(kRegThreads, NK >= 20 ? 1 : 2)
-spec_stats_kernel(const __grid_constant__ SpecParams<CAP> p) {
-  __shared__ RefSum red[2][kRegWarps];
-  __shared__ float4 cl_slot[kMaxCluster][2];
-  const uint32_t crank = cluster_ctarank();
-  const uint32_t csize = cluster_nctarank();
-  cluster_arrive_relaxed();  // phase A: every CTA of the cluster has started
+// ------------------------------------------ packed fp32 pairs (f32x2)
+// Each op is two IEEE round-to-nearest operations in one instruction.
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
+  float2 d;
+  asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
+      "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+  return d;
+}
+__device__ __forceinline__ float2 add2(float2 a, float2 b) {
+  float2 d;
+  asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+      "add.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return d;
+}
+__device__ __forceinline__ float2 sub2(float2 a, float2 b) {
+  float2 d;
+  asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+      "sub.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return d;
+}
+// ex2_ref on a pair: the same two roundings as ex2_ref, so the same bits
+__device__ __forceinline__ float2 ex2_ref2(float2 x, float2 ncf) {
+  const float2 a = fma2(x, make_float2(kLog2eHi, kLog2eHi), ncf);
+  const float2 b = fma2(x, make_float2(kLog2eLo, kLog2eLo), a);
+  return make_float2(fast_ex2(b.x), fast_ex2(b.y));
+}
 
-  const int n = blockIdx.x / csize;  // verify position
-  const int ui = spec_find_user<CAP>(p.q_off, p.B, n);
-  const int t = n - p.q_off[ui];
-  const int Li = p.q_off[ui + 1] - p.q_off[ui] - 1;
-  const bool has_q = t < Li;
-  const int wrow = p.l_off[ui] + t;
-  const T* zrow = static_cast<const T*>(p.z) + static_cast<size_t>(n) * p.V;
-  const T* wrow_p = static_cast<const T*>(p.w) + static_cast<size_t>(has_q ? wrow : 0) * p.V;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  int sb, se;
-  slice_bounds(p.nvec, crank, csize, sb, se);
-
-  pdl_wait_prior_grid();
-  pdl_launch_dependents();
-  uint4 rz[NK], rw[NK];
-  load_slice<NK>(reinterpret_cast<const uint8_t*>(zrow), sb, se, threadIdx.x, rz);
-  if (has_q) load_slice<NK>(reinterpret_cast<const uint8_t*>(wrow_p), sb, se, threadIdx.x, rw);
-  // rank 0 fetches the draft token's two logits now; they are used at the end
-  int d = -1;
-  float zd = 0.f, wd = 0.f;
-  if (crank == 0 && threadIdx.x == 0 && has_q) {
-    d = p.draft_tokens[wrow];
-    if (d >= 0 && d < p.V) {
-      zd = load_elem<T>(zrow, d);
-      wd = load_elem<T>(wrow_p, d);
+// Sum of 2^(x log2 e - c) over a lane's vectors k0 <= k < k0 + KG, k < nv:
+// pairs of logits in f32x2 arithmetic, Kahan over vectors on the pair.
+template <typename T, int NK, int KG>
+__device__ __forceinline__ FF lane_expsum(const uint4 (&r)[NK], int k0, int nv, float cf) {
+  const float2 ncf = make_float2(-cf, -cf);
+  float2 s = make_float2(0.f, 0.f), c = make_float2(0.f, 0.f);
+#pragma unroll
+  for (int k = k0; k < k0 + KG; ++k) {
+    if (k < nv) {
+      const uint32_t w[4] = {r[k].x, r[k].y, r[k].z, r[k].w};
+      float2 v;
+      if constexpr (sizeof(T) == 2) {
+        float2 e[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          e[j] = ex2_ref2(make_float2(__uint_as_float(w[j] << 16), __uint_as_float(w[j] & 0xFFFF0000u)), ncf);
+        v = add2(add2(e[0], e[1]), add2(e[2], e[3]));
+      } else {
+        const float2 e0 = ex2_ref2(make_float2(__uint_as_float(w[0]), __uint_as_float(w[1])), ncf);
+        const float2 e1 = ex2_ref2(make_float2(__uint_as_float(w[2]), __uint_as_float(w[3])), ncf);
+        v = add2(e0, e1);
+      }
+      // Kahan step on both halves
+      const float2 y = sub2(v, c);
+      const float2 t = add2(s, y);
+      c = sub2(sub2(t, s), y);
+      s = t;
     }
   }
-
-  RefSum az = thread_refsum<T, NK>(rz, sb, se, threadIdx.x);
-  RefSum aw{kEmptyRef, FF{0.f, 0.f}};
-  if (has_q) aw = thread_refsum<T, NK>(rw, sb, se, threadIdx.x);
-  az = warp_refsum(az);
-  aw = warp_refsum(aw);
-  if (lane == 0) {
-    red[0][warp] = az;
-    red[1][warp] = aw;
-  }
-  __syncthreads();
-  cluster_wait_acquire();  // phase A complete: rank 0 is running
-  if (threadIdx.x == 0) {
-    RefSum bz = red[0][0], bw = red[1][0];
-    for (int k = 1; k < kRegWarps; ++k) {
-      bz = refsum_add(bz, red[0][k]);
-      bw = refsum_add(bw, red[1][k]);
-    }
-    const uint32_t dst = dsmem_map(&cl_slot[crank][0], 0);
-    dsmem_st_f32x4(dst, __int_as_float(bz.c), bz.s.hi, bz.s.lo, 0.f);
-    dsmem_st_f32x4(dst + 16, __int_as_float(bw.c), bw.s.hi, bw.s.lo, 0.f);
-  }
-  cluster_arrive_release();  // phase B: slices delivered to rank 0
-  cluster_wait_acquire();
-  if (crank != 0 || threadIdx.x != 0) return;
-
-  RefSum fz{kEmptyRef, FF{0.f, 0.f}}, fw{kEmptyRef, FF{0.f, 0.f}};
-  for (uint32_t k = 0; k < csize; ++k) {
-    const float4 a = cl_slot[k][0], b = cl_slot[k][1];
-    fz = refsum_add(fz, RefSum{__float_as_int(a.x), FF{a.y, a.z}});
-    fw = refsum_add(fw, RefSum{__float_as_int(b.x), FF{b.y, b.z}});
-  }
-  SpecStat st;
-  st.sz = static_cast<double>(fz.s.hi) + static_cast<double>(fz.s.lo);
-  st.sw = static_cast<double>(fw.s.hi) + static_cast<double>(fw.s.lo);
-  st.cz = fz.c;
-  st.cw = fw.c;
-  st.pad0 = st.pad1 = 0;
-  static_cast<SpecStat*>(p.stats)[n] = st;
-  float pd = 0.f, qd = 0.f;
-  unsigned char flag = 0;
-  if (has_q) {
-    if (d >= 0 && d < p.V) {
-      const float ez = ex2_ref(zd, st.cz);
-      const float ew = ex2_ref(wd, st.cw);
-      pd = ez * (1.f / static_cast<float>(st.sz));
-      qd = ew * (1.f / static_cast<float>(st.sw));
-      // u * q(d) < p(d), i.e. u * ew * sz < ez * sw (products in fp64, no division)
-      flag = static_cast<double>(p.uniforms[2 * n]) * static_cast<double>(ew) * st.sz <
-                     static_cast<double>(ez) * st.sw ? 1 : 0;
-    } else {
-      atomicOr(p.status, kDevErrBadToken);
-    }
-  }
-  p.flags[n] = flag;
-  if (p.draft_probs) reinterpret_cast<float2*>(p.draft_probs)[n] = make_float2(pd, qd);
+  // the two halves' compensated sums, added exactly
+  return ff_add(FF{s.x, -c.x}, FF{s.y, -c.y});
 }
 
 // Sampling weights of one vector: (p - q)^+ up to the common factor 1/sz
-// (residual), or p up to 1/sz (bonus).  Explicit rounding, so every
-// evaluation of the same vector yields the same bits.
+// (residual), or p up to 1/sz.  Explicit rounding, so every evaluation of the
+// same vector yields the same bits.
 template <typename T>
 __device__ __forceinline__ void vec_weights(const uint4& rz, const uint4& rw, bool residual, int cz, int cw,
                                             float khi, float klo, float (&wt)[Vec16<T>::N]) {
@@ -341,244 +343,419 @@ __device__ __forceinline__ float vec_sum(const float (&wt)[N]) {
   return s;
 }
 
-// ------------------------------------------------------------------ pass 2
-template <typename T, int NK, int CAP>
-__global__ void __launch_bounds__(kRegThreads, 1)
-spec_sample_kernel(const __grid_constant__ SpecParams<CAP> p) {
+// inclusive fp32 scan over the lanes
+__device__ __forceinline__ float warp_scan_f32(float v, int lane) {
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float y = __shfl_up_sync(0xffffffffu, v, o);
+    if (lane >= o) v = __fadd_rn(v, y);
+  }
+  return v;
+}
+
+// Totals of one segment's weights in token order: step k covers the 32
+// consecutive vectors vb + k * 32 + (0..31) (a group); a group total is the
+// last lane of an fp32 scan over the lanes, groups add up in float-float.  tr
+// is the residual's total (p's when not residual) and tp p's.  Bit-identical
+// to the descent's recomputation from vec_weights and vec_sum.
+template <typename T, int NK>
+__device__ __forceinline__ void segment_totals(const uint4 (&rz)[NK], const uint4 (&rw)[NK], int nv, bool residual,
+                                               const WRef& st, int lane, FF& tr, FF& tp) {
   constexpr int N = Vec16<T>::N;
-  __shared__ float gsum[NK * kRegWarps];      // group totals, group g = step k * warps + warp
-  __shared__ float gpre[NK * kRegWarps][2];   // float-float inclusive prefix of the groups
-  __shared__ float slice_sum[2][kMaxCluster][2];
-  __shared__ int s_off, s_a, s_cnt[kRegWarps];
-  __shared__ int s_sel[3];
-  __shared__ float s_rem[2];
-  __shared__ float s_k[2];
-  const uint32_t crank = cluster_ctarank();
-  const uint32_t csize = cluster_nctarank();
-  cluster_arrive_relaxed();  // phase A: every CTA has started
-
-  const int ui = blockIdx.x / csize;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  pdl_wait_prior_grid();
-  pdl_launch_dependents();
-
-  // a_i and the packed offset sum_{j<i} (a_j + 1), by warp ballots
-  int cnt = 0;
-  for (int j = warp; j < ui; j += kRegWarps) cnt += accepted_prefix<CAP>(p, j, lane) + 1;
-  if (lane == 0) s_cnt[warp] = cnt;
-  if (warp == 0) {
-    const int a = accepted_prefix<CAP>(p, ui, lane);
-    if (lane == 0) s_a = a;
-  }
-  __syncthreads();
-  const int q0 = p.q_off[ui], l0 = p.l_off[ui];
-  const int Li = p.q_off[ui + 1] - q0 - 1;
-  if (threadIdx.x == 0) {
-    int o = 0;
-    for (int k = 0; k < kRegWarps; ++k) o += s_cnt[k];
-    s_off = o;
-    // scale of q relative to p in the residual, split into two floats
-    const SpecStat st0 = static_cast<const SpecStat*>(p.stats)[q0 + s_a];
-    const double kd = s_a < Li ? st0.sz / st0.sw : 0.0;
-    const float kh = static_cast<float>(kd);
-    s_k[0] = kh;
-    s_k[1] = static_cast<float>(kd - static_cast<double>(kh));
-  }
-  __syncthreads();
-  const int a = s_a, off = s_off;
-  if (crank == 0) {
-    for (int k = threadIdx.x; k < a; k += kRegThreads) p.out_tokens[off + k] = p.draft_tokens[l0 + k];
-    if (threadIdx.x == 0) {
-      p.accept_len[ui] = a;
-      p.out_offsets[ui] = off;
-      if (ui == p.B - 1) p.out_offsets[p.B] = off + a + 1;
-    }
-  }
-
-  // the rows of position a, this CTA's slice, into registers
-  const int n = q0 + a;
-  bool residual = a < Li;
-  const SpecStat st = static_cast<const SpecStat*>(p.stats)[n];
-  const uint8_t* zrow = reinterpret_cast<const uint8_t*>(static_cast<const T*>(p.z) + static_cast<size_t>(n) * p.V);
-  const uint8_t* wrow =
-      reinterpret_cast<const uint8_t*>(static_cast<const T*>(p.w) + static_cast<size_t>(residual ? l0 + a : 0) * p.V);
-  int sb, se;
-  slice_bounds(p.nvec, crank, csize, sb, se);
-  uint4 rz[NK], rw[NK];
-  load_slice<NK>(zrow, sb, se, threadIdx.x, rz);
-  if (residual) load_slice<NK>(wrow, sb, se, threadIdx.x, rw);
-  const float khi = s_k[0], klo = s_k[1];
-  const float u = p.uniforms[2 * n + 1];
-
-  // one pass per candidate distribution: the residual, then p if it is empty
-  constexpr int G = NK * kRegWarps;  // groups of this CTA, in token order (step k, warp)
-  for (int round = 0; round < 2; ++round) {
+  tr = FF{0.f, 0.f};
+  tp = FF{0.f, 0.f};
 #pragma unroll
-    for (int k = 0; k < NK; ++k) {
-      float ls = 0.f;
-      if (sb + k * kRegThreads + static_cast<int>(threadIdx.x) < se) {
-        float wt[N];
-        vec_weights<T>(rz[k], rw[k], residual, st.cz, st.cw, khi, klo, wt);
-        ls = vec_sum<N>(wt);
-      }
-      float incl = ls;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const float y = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl = __fadd_rn(incl, y);
-      }
-      if (lane == 31) gsum[k * kRegWarps + warp] = incl;
-    }
-    __syncthreads();
-    // warp 0: float-float prefix over the groups; the last one is the slice total
-    if (warp == 0) {
-      FF carry{0.f, 0.f};
-      for (int g0 = 0; g0 < G; g0 += 32) {
-        const int g = g0 + lane;
-        FF v{g < G ? gsum[g] : 0.f, 0.f};
-        v = ff_add(warp_ff_scan(v, lane), carry);
-        if (g < G) {
-          gpre[g][0] = v.hi;
-          gpre[g][1] = v.lo;
-        }
-        carry.hi = __shfl_sync(0xffffffffu, v.hi, 31);
-        carry.lo = __shfl_sync(0xffffffffu, v.lo, 31);
-      }
-      if (lane == 0) {
-        if (round == 0) cluster_wait_acquire();  // phase A complete: all CTAs running
-        for (uint32_t r = 0; r < csize; ++r)
-          dsmem_st_f32x2(dsmem_map(&slice_sum[round][crank][0], r), carry.hi, carry.lo);
-      }
-    }
-    if (round == 0 && warp != 0) cluster_wait_acquire();
-    if (round == 0 && warp == 0 && lane != 0) cluster_wait_acquire();
-    cluster_arrive_release();
-    cluster_wait_acquire();
-
-    // thread 0 finds the slice and group holding u * total (if rounding
-    // leaves none: the last positive weight at every level) and publishes
-    // them with the remainder below the group; all in float-float
-    if (threadIdx.x == 0) {
-      FF total{0.f, 0.f};
-      for (uint32_t r = 0; r < csize; ++r) total = ff_add(total, FF{slice_sum[round][r][0], slice_sum[round][r][1]});
-      int mode = 0;  // 0: crossing, 1: last positive weight, 2: empty distribution
-      int cs = static_cast<int>(csize) - 1;
-      FF rem{0.f, 0.f};
-      if (!(total.hi > 0.f)) {
-        mode = 2;
-      } else {
-        rem = ff_mul_f(total, u);
-        mode = 1;
-        for (uint32_t r = 0; r < csize; ++r) {
-          const FF sl{slice_sum[round][r][0], slice_sum[round][r][1]};
-          if (ff_gt(sl, rem)) { cs = static_cast<int>(r); mode = 0; break; }
-          rem = ff_sub(rem, sl);
-        }
-        if (mode == 1)
-          while (cs > 0 && !(slice_sum[round][cs][0] > 0.f)) --cs;
-      }
-      s_sel[0] = mode;
-      s_sel[1] = cs;
-      s_rem[0] = rem.hi;
-      s_rem[1] = rem.lo;
-    }
-    __syncthreads();
-    int mode = s_sel[0];
-    if (mode == 2) {
-      if (residual) {  // no residual mass left: fall back to p at this position
-        residual = false;
-        continue;
-      }
-      return;  // p always has mass for finite logits
-    }
-    if (s_sel[1] != static_cast<int>(crank)) return;
-    // warp 0 of the chosen slice: first group whose prefix exceeds the remainder
-    if (warp == 0) {
-      const FF rem{s_rem[0], s_rem[1]};
-      int gsel = -1;
-      if (mode == 0) {
-        for (int g0 = 0; g0 < G && gsel < 0; g0 += 32) {
-          const int g = g0 + lane;
-          const bool hit = g < G && ff_gt(FF{gpre[g][0], gpre[g][1]}, rem);
-          const unsigned bal = __ballot_sync(0xffffffffu, hit);
-          if (bal) gsel = g0 + __ffs(bal) - 1;
-        }
-      }
-      if (gsel < 0) {  // rounding: the last group with mass
-        mode = 1;
-        int lastg = 0;
-        for (int g0 = 0; g0 < G; g0 += 32) {
-          const int g = g0 + lane;
-          const unsigned bal = __ballot_sync(0xffffffffu, g < G && gsum[g] > 0.f);
-          if (bal) lastg = g0 + 31 - __clz(bal);
-        }
-        gsel = lastg;
-      }
-      if (lane == 0) {
-        FF rg = rem;
-        if (gsel > 0) rg = ff_sub(rem, FF{gpre[gsel - 1][0], gpre[gsel - 1][1]});
-        s_sel[0] = mode;
-        s_sel[2] = gsel;
-        s_rem[0] = rg.hi;
-        s_rem[1] = rg.lo;
-      }
-    }
-    __syncthreads();
-    mode = s_sel[0];
-    const int gk = s_sel[2] / kRegWarps, gw = s_sel[2] % kRegWarps;
-    if (gw != warp) return;
-    bool last = mode == 1;
-    const FF remg{s_rem[0], s_rem[1]};
-
-    // recompute group (gk, gw) exactly as in the totals and descend to the token
-    const int v = sb + gk * kRegThreads + static_cast<int>(threadIdx.x);
-    float wt[N];
-#pragma unroll
-    for (int e = 0; e < N; ++e) wt[e] = 0.f;
-    uint4 mz = rz[0], mw = rw[0];
-#pragma unroll
-    for (int k = 1; k < NK; ++k)
-      if (k == gk) { mz = rz[k]; mw = rw[k]; }
-    if (v < se) vec_weights<T>(mz, mw, residual, st.cz, st.cw, khi, klo, wt);
-    const float ls = vec_sum<N>(wt);
-    float incl = ls;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const float y = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl = __fadd_rn(incl, y);
-    }
-    int ln = 0;
-    if (!last) {
-      const unsigned hit = __ballot_sync(0xffffffffu, ff_gt(FF{incl, 0.f}, remg));
-      ln = hit ? __ffs(hit) - 1 : -1;
-      if (ln < 0) last = true;
-    }
-    if (last) {
-      const unsigned pos = __ballot_sync(0xffffffffu, ls > 0.f);
-      ln = pos ? 31 - __clz(pos) : 0;
-    }
-    float ex = __shfl_up_sync(0xffffffffu, incl, 1);
-    if (lane == 0) ex = 0.f;
-    if (lane == ln) {
-      const FF reml = ff_sub(remg, FF{ex, 0.f});
-      int k = -1;
-      float c = 0.f;
-      if (!last) {
+  for (int k = 0; k < NK; ++k) {
+    float sr = 0.f, sp = 0.f;
+    if (k < nv) {
+      float xz[N];
+      Vec16<T>::unpack(rz[k], xz);
+      if (residual) {
+        float xw[N];
+        Vec16<T>::unpack(rw[k], xw);
 #pragma unroll
         for (int e = 0; e < N; ++e) {
-          c = __fadd_rn(c, wt[e]);
-          if (k < 0 && ff_gt(FF{c, 0.f}, reml)) k = e;
+          const float ez = ex2_ref(xz[e], st.cz);
+          const float ew = ex2_ref(xw[e], st.cw);
+          const float q = __fmaf_rn(ew, st.khi, __fmul_rn(ew, st.klo));
+          sr = __fadd_rn(sr, fmaxf(__fsub_rn(ez, q), 0.f));
+          sp = __fadd_rn(sp, ez);
+        }
+      } else {
+#pragma unroll
+        for (int e = 0; e < N; ++e) sp = __fadd_rn(sp, ex2_ref(xz[e], st.cz));
+      }
+    }
+    const float gp = __shfl_sync(0xffffffffu, warp_scan_f32(sp, lane), 31);
+    tp = ff_add(tp, FF{gp, 0.f});
+    if (residual) {
+      const float gr = __shfl_sync(0xffffffffu, warp_scan_f32(sr, lane), 31);
+      tr = ff_add(tr, FF{gr, 0.f});
+    }
+  }
+  if (!residual) tr = tp;
+}
+
+// ----------------------------------------------------- position decision
+// Run by the warp that delivered the last segment of position q0 + t of user
+// ui: row sums, p_t(d), q_t(d), the acceptance decision; the user's last
+// decided position also writes a_i.
+template <int CAP>
+__device__ __forceinline__ void decide_position(const SpecParams<CAP>& p, int ui, int t, int lane) {
+  const int q0 = p.q_off[ui];
+  const int Li = p.q_off[ui + 1] - q0 - 1;
+  const int n = q0 + t, l = p.l_off[ui] + t;
+  const bool has_q = t < Li;
+  const float4* pz = p.part1 + static_cast<size_t>(n) * p.nseg1;
+  const float4* pw = p.part1 + static_cast<size_t>(p.sum_t + l) * p.nseg1;
+  // every load first: the draft token's logits, left by the rows' first
+  // segments (NaN: d outside [0, V)), and both rows' segment partials
+  float zd = 0.f, wd = 0.f;
+  if (has_q && lane == 0) {
+    zd = __ldcg(&pz->w);
+    wd = __ldcg(&pw->w);
+  }
+  RefSum az{kEmptyRef, FF{0.f, 0.f}}, aw{kEmptyRef, FF{0.f, 0.f}};
+#pragma unroll 2
+  for (int sg = lane; sg < p.nseg1; sg += 32) {
+    const float4 vz = __ldcg(pz + sg);
+    const float4 vw = has_q ? __ldcg(pw + sg) : make_float4(__int_as_float(kEmptyRef), 0.f, 0.f, 0.f);
+    az = refsum_add(az, RefSum{__float_as_int(vz.x), FF{vz.y, vz.z}});
+    aw = refsum_add(aw, RefSum{__float_as_int(vw.x), FF{vw.y, vw.z}});
+  }
+  az = warp_refsum(az);
+  if (has_q) aw = warp_refsum(aw);
+  if (lane == 0) {
+    p.counters[n] = 0u;
+    SpecStat st;
+    st.sz = static_cast<double>(az.s.hi) + static_cast<double>(az.s.lo);
+    st.cz = az.c;
+    st.sw = 0.0;
+    st.cw = kEmptyRef;
+    st.khi = st.klo = 0.f;
+    float pd = 0.f, qd = 0.f;
+    unsigned char flag = 0;
+    if (has_q) {
+      st.sw = static_cast<double>(aw.s.hi) + static_cast<double>(aw.s.lo);
+      st.cw = aw.c;
+      // sz / sw in float-float: q1 = zh / wh, then the remainder's quotient
+      const float q1 = __fdiv_rn(az.s.hi, aw.s.hi);
+      float r = __fmaf_rn(-q1, aw.s.hi, az.s.hi);
+      r = __fmaf_rn(-q1, aw.s.lo, __fadd_rn(r, az.s.lo));
+      const float q2 = __fdiv_rn(r, aw.s.hi);
+      st.khi = __fadd_rn(q1, q2);
+      st.klo = __fsub_rn(q2, __fsub_rn(st.khi, q1));
+      if (zd == zd && wd == wd) {
+        const float ez = ex2_ref(zd, st.cz);
+        const float ew = ex2_ref(wd, st.cw);
+        pd = ez * (1.f / static_cast<float>(st.sz));
+        qd = ew * (1.f / static_cast<float>(st.sw));
+        // u * q(d) < p(d), i.e. u * ew * sz < ez * sw (products in fp64, no division)
+        flag = static_cast<double>(p.uniforms[2 * n]) * static_cast<double>(ew) * st.sz <
+                       static_cast<double>(ez) * st.sw ? 1 : 0;
+      } else {
+        atomicOr(p.status, kDevErrBadToken);
+      }
+    }
+    static_cast<SpecStat*>(p.stats)[n] = st;
+    if (p.draft_probs) reinterpret_cast<float2*>(p.draft_probs)[n] = make_float2(pd, qd);
+    // the user's decision word: one arrival, and bit t if d_{t+1} is accepted;
+    // the last of the user's L_i + 1 positions reads a_i off the sum
+    unsigned long long* word = reinterpret_cast<unsigned long long*>(p.counters + kCntUser1) + ui;
+    const unsigned long long add = (1ull << 32) | (flag ? (1ull << t) : 0ull);
+    const unsigned long long now = atomicAdd(word, add) + add;
+    if (static_cast<int>(now >> 32) == Li + 1) {
+      p.accept_len[ui] = min(__ffs(~static_cast<unsigned>(now)) - 1, Li);
+      *word = 0ull;
+    }
+  }
+}
+
+// ------------------------------------------------------------------ pass 1
+template <typename T, int NK, int CAP>
+__global__ void __launch_bounds__(kRegThreads, 2)
+spec_stats_kernel(const __grid_constant__ SpecParams<CAP> p) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int item = blockIdx.x * kRegWarps + warp;
+  pdl_wait_prior_grid();
+  pdl_launch_dependents();
+  if (item >= p.n_items1) return;
+  const int row = item / p.nseg1;
+  const int s = item - row * p.nseg1;
+  const bool is_w = row >= p.sum_t;  // rows: every z_t, then every w_t
+  const int ui = is_w ? spec_find_user<CAP>(p.l_off, p.B, row - p.sum_t) : spec_find_user<CAP>(p.q_off, p.B, row);
+  const int q0 = p.q_off[ui];
+  const int Li = p.q_off[ui + 1] - q0 - 1;
+  const int t = is_w ? row - p.sum_t - p.l_off[ui] : row - q0;
+  const int n = q0 + t, l = p.l_off[ui] + t;
+  const bool has_q = t < Li;
+  const T* rowp = is_w ? static_cast<const T*>(p.w) + static_cast<size_t>(l) * p.V
+                       : static_cast<const T*>(p.z) + static_cast<size_t>(n) * p.V;
+  const int vb = s * (32 * NK);
+  const int nv = lane_vectors(p.nvec, vb, lane, NK);
+  uint4 r[NK];
+  load_segment<NK>(rowp, vb, lane, nv, r);
+  // the draft token's logit, fetched by lane 0 of the row's first segment
+  float xd = 0.f;
+  if (s == 0 && lane == 0 && has_q) {
+    const int d = p.draft_tokens[l];
+    xd = d >= 0 && d < p.V ? load_elem<T>(rowp, d) : __int_as_float(0x7fc00000);
+  }
+  // groups of four vectors, each with its own warp reference, so that the
+  // first group's exponentials overlap the later groups' loads
+  constexpr int KG = NK < 4 ? NK : 4;
+  RefSum tot{kEmptyRef, FF{0.f, 0.f}};
+#pragma unroll
+  for (int k0 = 0; k0 < NK; k0 += KG) {
+    const float m = lane_max<T, NK, KG>(r, k0, nv);
+    int c = m > -INFINITY ? static_cast<int>(fminf(fmaxf(ceilf(m * kLog2e), -1048576.f), 1048576.f)) : kEmptyRef;
+    c = __reduce_max_sync(0xffffffffu, c);
+    if (c != kEmptyRef) tot = refsum_add(tot, RefSum{c, lane_expsum<T, NK, KG>(r, k0, nv, static_cast<float>(c))});
+  }
+  const int c = tot.c;  // the same in every lane
+  const FF sum = warp_ff_sum(tot.s);
+  unsigned cnt = 0;
+  if (lane == 0) {
+    p.part1[item] = make_float4(__int_as_float(c), sum.hi, sum.lo, xd);
+    cnt = counter_arrive(p.counters + n);
+  }
+  __syncwarp();
+  cnt = __shfl_sync(0xffffffffu, cnt, 0);
+  if (cnt != static_cast<unsigned>(p.nseg1 * (has_q ? 2 : 1))) return;
+  decide_position<CAP>(p, ui, t, lane);
+}
+
+// ------------------------------------------------------------------ pass 2
+// Run by the warp that delivered the last segment of user ui: packed output
+// offset, accepted drafts, then the inverse-CDF descent to the emitted token.
+template <typename T, int NK, int CAP>
+__device__ __forceinline__ void descend(const SpecParams<CAP>& p, int ui, int a, bool residual, const WRef& st,
+                                        const T* zrow, const T* wrow, int lane) {
+  constexpr int N = Vec16<T>::N;
+  const int q0 = p.q_off[ui], l0 = p.l_off[ui];
+  const int n = q0 + a;
+  if (lane == 0) p.counters[kCntUser2 + ui] = 0u;
+  int o = 0;
+  for (int j = lane; j < ui; j += 32)
+    o += min(max(p.accept_len[j], 0), p.q_off[j + 1] - p.q_off[j] - 1) + 1;
+  const int off = __reduce_add_sync(0xffffffffu, o);
+  for (int k = lane; k < a; k += 32) p.out_tokens[off + k] = p.draft_tokens[l0 + k];
+  if (lane == 0) {
+    p.out_offsets[ui] = off;
+    if (ui == p.B - 1) p.out_offsets[p.B] = off + a + 1;
+  }
+  const float u = p.uniforms[2 * n + 1];
+  const float4* part = p.part2 + static_cast<size_t>(ui) * p.nseg2;
+  const int per = (p.nseg2 + 31) >> 5;  // lane j owns segments [j per, (j + 1) per)
+  const int s0 = lane * per;
+  // a run of up to kRun segments per lane is held in registers as its
+  // running float-float sums (the same additions in the same order as the
+  // lane's total), so the walk below compares them all at once
+  constexpr int kRun = 16;
+  const bool in_regs = per <= kRun;
+  // mode 0: the residual; mode 1: p (the bonus position, or an empty residual)
+  for (int mode = residual ? 0 : 1; mode < 2; ++mode) {
+    FF pre[kRun];
+    FF ls{0.f, 0.f};
+    if (in_regs) {
+      float2 v[kRun];
+#pragma unroll
+      for (int i = 0; i < kRun; ++i) {
+        const int sg = s0 + i;
+        v[i] = i < per && sg < p.nseg2 ? __ldcg(reinterpret_cast<const float2*>(part + sg) + mode)
+                                       : make_float2(0.f, 0.f);
+      }
+#pragma unroll
+      for (int i = 0; i < kRun; ++i) {
+        ls = ff_add(ls, FF{v[i].x, v[i].y});
+        pre[i] = ls;
+      }
+    } else {
+      for (int i = 0; i < per; ++i) {
+        const int sg = s0 + i;
+        if (sg < p.nseg2) {
+          const float2 v = __ldcg(reinterpret_cast<const float2*>(part + sg) + mode);
+          ls = ff_add(ls, FF{v.x, v.y});
         }
       }
-      if (k < 0) {
-        for (int e = N - 1; e >= 0; --e)
-          if (wt[e] > 0.f) { k = e; break; }
-        if (k < 0) k = 0;
+    }
+    const FF incl = warp_ff_scan(ls, lane);
+    const FF total = ff_shfl(incl, 31);
+    if (!(total.hi > 0.f)) continue;
+    const FF target = ff_mul_f(total, u);
+    // level 1: the lane whose run of segments holds the target (if rounding
+    // leaves none: the last positive mass at every level)
+    const unsigned hit = __ballot_sync(0xffffffffu, ff_gt(incl, target));
+    bool last = hit == 0;
+    const int ln = last ? 31 - __clz(__ballot_sync(0xffffffffu, ls.hi > 0.f)) : __ffs(hit) - 1;
+    const FF rem = ff_sub(target, ff_shfl(warp_ff_exclusive(incl, lane), ln));
+    int sel = -1;
+    FF rs{0.f, 0.f};
+    if (lane == ln) {
+      int lastpos = -1;
+      if (in_regs) {
+        FF prev{0.f, 0.f};
+#pragma unroll
+        for (int i = 0; i < kRun; ++i) {
+          if (sel < 0 && !last && ff_gt(pre[i], rem)) {
+            sel = s0 + i;
+            rs = ff_sub(rem, prev);
+          }
+          if (pre[i].hi != prev.hi || pre[i].lo != prev.lo) lastpos = s0 + i;
+          prev = pre[i];
+        }
+      } else {
+        FF run{0.f, 0.f};
+        for (int i = 0; i < per; ++i) {
+          const int sg = s0 + i;
+          if (sg >= p.nseg2) break;
+          const float2 v = __ldcg(reinterpret_cast<const float2*>(part + sg) + mode);
+          const FF x{v.x, v.y};
+          const FF nx = ff_add(run, x);
+          if (!last && ff_gt(nx, rem)) {
+            sel = sg;
+            rs = ff_sub(rem, run);
+            break;
+          }
+          if (x.hi > 0.f) lastpos = sg;
+          run = nx;
+        }
       }
-      p.out_tokens[off + a] = v * N + k;
+      if (sel < 0) {
+        sel = lastpos;
+        last = true;
+      }
+    }
+    sel = min(max(__shfl_sync(0xffffffffu, sel, ln), 0), p.nseg2 - 1);
+    last = __shfl_sync(0xffffffffu, last ? 1 : 0, ln) != 0;
+    rs = ff_shfl(rs, ln);
+    // level 2: the segment's groups, recomputed exactly as in its totals
+    const int vb = sel * (32 * NK);
+    const int nv = lane_vectors(p.nvec, vb, lane, NK);
+    uint4 rz[NK], rw[NK];
+    load_segment<NK>(zrow, vb, lane, nv, rz);
+    load_segment<NK>(wrow, vb, lane, residual ? nv : 0, rw);
+    float vs[NK], gin[NK];
+#pragma unroll
+    for (int k = 0; k < NK; ++k) {
+      vs[k] = 0.f;
+      if (k < nv) {
+        float wt[N];
+        vec_weights<T>(rz[k], rw[k], mode == 0, st.cz, st.cw, st.khi, st.klo, wt);
+        vs[k] = vec_sum<N>(wt);
+      }
+      gin[k] = warp_scan_f32(vs[k], lane);
+    }
+    int kk = -1, lastk = -1;
+    FF rg{0.f, 0.f}, run{0.f, 0.f};
+#pragma unroll
+    for (int k = 0; k < NK; ++k) {
+      const float g = __shfl_sync(0xffffffffu, gin[k], 31);
+      const FF nx = ff_add(run, FF{g, 0.f});
+      if (kk < 0 && !last && ff_gt(nx, rs)) {
+        kk = k;
+        rg = ff_sub(rs, run);
+      }
+      if (g > 0.f) lastk = k;
+      run = nx;
+    }
+    if (kk < 0) {
+      kk = max(lastk, 0);
+      last = true;
+    }
+    // level 3: the lane of group kk, then the token inside its vector
+    float ik = 0.f, vk = 0.f;
+    uint4 mz = rz[0], mw = rw[0];
+#pragma unroll
+    for (int k = 0; k < NK; ++k)
+      if (k == kk) {
+        ik = gin[k];
+        vk = vs[k];
+        mz = rz[k];
+        mw = rw[k];
+      }
+    int ln2 = -1;
+    if (!last) {
+      const unsigned h2 = __ballot_sync(0xffffffffu, ff_gt(FF{ik, 0.f}, rg));
+      if (h2) ln2 = __ffs(h2) - 1;
+      else last = true;
+    }
+    if (last) {
+      const unsigned pos = __ballot_sync(0xffffffffu, vk > 0.f);
+      ln2 = pos ? 31 - __clz(pos) : 0;
+    }
+    float ex = __shfl_up_sync(0xffffffffu, ik, 1);
+    if (lane == 0) ex = 0.f;
+    const FF rl = ff_sub(rg, FF{__shfl_sync(0xffffffffu, ex, ln2), 0.f});
+    if (lane == ln2) {
+      float wt[N];
+#pragma unroll
+      for (int e = 0; e < N; ++e) wt[e] = 0.f;
+      if (kk < nv) vec_weights<T>(mz, mw, mode == 0, st.cz, st.cw, st.khi, st.klo, wt);
+      int es = -1;
+      if (!last) {
+        float cum = 0.f;
+#pragma unroll
+        for (int e = 0; e < N; ++e) {
+          cum = __fadd_rn(cum, wt[e]);
+          if (es < 0 && ff_gt(FF{cum, 0.f}, rl)) es = e;
+        }
+      }
+      if (es < 0) {
+#pragma unroll
+        for (int e = 0; e < N; ++e)
+          if (wt[e] > 0.f) es = e;
+      }
+      if (es < 0) es = 0;
+      p.out_tokens[off + a] = min((vb + kk * 32 + lane) * N + es, p.V - 1);
     }
     return;
   }
+  if (lane == 0) p.out_tokens[off + a] = 0;  // no mass at all: every logit -inf
+}
+
+template <typename T, int NK, int CAP>
+__global__ void __launch_bounds__(kRegThreads, 2)
+spec_sample_kernel(const __grid_constant__ SpecParams<CAP> p) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int item = blockIdx.x * kRegWarps + warp;
+  pdl_wait_prior_grid();
+  pdl_launch_dependents();
+  if (item >= p.n_items2) return;
+  const int ui = item / p.nseg2;
+  const int s = item - ui * p.nseg2;
+  const int q0 = p.q_off[ui], l0 = p.l_off[ui];
+  const int Li = p.q_off[ui + 1] - q0 - 1;
+  // a_i and the weight references of all the user's positions, fetched together
+  const int a_raw = p.accept_len[ui];
+  int4 ref4 = make_int4(0, 0, 0, 0);
+  if (lane <= Li) ref4 = reinterpret_cast<const int4*>(static_cast<const SpecStat*>(p.stats) + q0 + lane)[1];
+  const int a = min(max(a_raw, 0), Li);  // (clamped: written by the stats kernel)
+  const int n = q0 + a;
+  const bool residual = a < Li;
+  WRef st;
+  st.cz = __shfl_sync(0xffffffffu, ref4.x, a);
+  st.cw = __shfl_sync(0xffffffffu, ref4.y, a);
+  st.khi = __int_as_float(__shfl_sync(0xffffffffu, ref4.z, a));
+  st.klo = __int_as_float(__shfl_sync(0xffffffffu, ref4.w, a));
+  const T* zrow = static_cast<const T*>(p.z) + static_cast<size_t>(n) * p.V;
+  const T* wrow = residual ? static_cast<const T*>(p.w) + static_cast<size_t>(l0 + a) * p.V : zrow;
+  const int vb = s * (32 * NK);
+  const int nv = lane_vectors(p.nvec, vb, lane, NK);
+  uint4 rz[NK], rw[NK];
+  load_segment<NK>(zrow, vb, lane, nv, rz);
+  load_segment<NK>(wrow, vb, lane, residual ? nv : 0, rw);
+  FF R, P;
+  segment_totals<T, NK>(rz, rw, nv, residual, st, lane, R, P);
+  unsigned cnt = 0;
+  if (lane == 31) {
+    p.part2[item] = make_float4(R.hi, R.lo, P.hi, P.lo);
+    cnt = counter_arrive(p.counters + kCntUser2 + ui);
+  }
+  __syncwarp();
+  cnt = __shfl_sync(0xffffffffu, cnt, 31);
+  if (cnt != static_cast<unsigned>(p.nseg2)) return;
+  descend<T, NK, CAP>(p, ui, a, residual, st, zrow, wrow, lane);
 }
 
 }  // namespace dipsd
