@@ -37,6 +37,8 @@ struct AttnParams {
   float2* part_ml;  // per partial row: (running max in log2 units, sum)
   float* part_o;    // per partial row: D unnormalised outputs
   unsigned* status;
+  int cluster;  // > 1: the nsplit == cluster splits of a row block and head
+                // form one thread-block cluster and merge in shared memory
   int B, Hq, Hkv, G, max_blocks;
   int n_items, n_merge;
   float scale_log2;  // softmax_scale * log2(e)

@@ -1,26 +1,39 @@
 // verify_attention on the 5th-generation tensor cores (tcgen05 + TMEM).
 //
-// Same work decomposition and output contract as verify_attention_kernel
-// (attention.cuh): one CTA per (user i, KV head h, row block, KV split);
+// Work decomposition: one CTA per (user i, KV head h, row block, KV split);
 // rows r = t*G + g pack the G query heads of the KV group and the T_i verify
 // tokens (Sec. II-A stage 2: all L_i+1 tokens of a user are verified in one
 // pass), so each K/V byte brought on chip serves every row.
 //
 // Roles (6 warps):
-//   warp 0      TMA producer: 4-D tensor-map loads of the user's pages into
-//               a 4-stage ring of 64-token K and V tiles (128-byte swizzle);
-//               page ids are fetched 32 at a time, one per lane, a group
-//               ahead, and a tile's 16 boxes go out from 16 lanes at once.
-//   warp 1      allocates TMEM; one thread issues tcgen05.mma:
-//                 S[b] = Q K^T   (M=128 rows, N=64 keys, K=16 per instruction)
-//                 O   += P V     (two N=64 column halves of head_dim)
-//               and commits completions to mbarriers.
-//   warps 2..5  one query row per thread (TMEM lane = row): load S with
+//   warp 0      TMA producer into a ring of kStages 64-token K tiles and a
+//               ring of as many V tiles (128-byte swizzle).  K: one box per
+//               page and 64-column half (2 KB), stored half after half, so a
+//               half is 64 rows at the uniform 1024-byte stride one N=64
+//               product needs.  V: one box per page (4 KB at D = 128, both
+//               halves through a 5-D tensor map whose third dimension steps
+//               128 bytes), stored page after page.  K and V stages are
+//               released separately: K once its Q K^T has run, V after its
+//               P V.  Page ids are fetched 32 at a time, one per lane, a
+//               group ahead.
+//   warp 1      allocates TMEM; one thread issues tcgen05.mma as operands
+//               become ready (no fixed order between the two products):
+//                 S[b] = Q K^T      (A = Q from shared memory, M=128, N=64)
+//                 O   += P[b] V     (A = P from tensor memory; a 16-key step
+//                                    is one page of V; two N=64 halves)
+//   warps 2..5  one query row per thread (TMEM lane = row): load S[b] with
 //               tcgen05.ld, causal mask, online softmax in log2 units with a
 //               lazy rescale (O in TMEM is rescaled only when a row maximum
-//               grows by more than 2^8), write P as bf16 into a swizzled
-//               shared buffer, and finally read O back for the output.
-// TMEM columns: S double buffer [0,64) [64,128), O [128, 128+D).
+//               grows by more than 2^8), write P as bf16 pairs into the first
+//               32 columns of S[b] with tcgen05.st, and finally read O back.
+// KV splits: either each split writes (m, l, O) rows to global memory for
+// verify_attention_merge_kernel, or (p.cluster > 1) the splits of one row
+// block and head run as one thread-block cluster: the other ranks push their
+// rows into rank 0's drained rings through distributed shared memory and
+// rank 0 merges them with its own O straight from TMEM.
+// TMEM columns: S/P double buffer [0,64) [64,128), O [128, 128+D).  Shared
+// memory holds Q and the two rings (P never leaves tensor memory), which is
+// what leaves room for kStages tiles of K and of V in flight.
 #pragma once
 
 #include "attention.cuh"
@@ -29,7 +42,6 @@
 namespace dipsd {
 
 constexpr int kTcThreads = 192;
-constexpr int kTcStages = 4;
 constexpr int kTcTile = 64;                // keys per tile
 constexpr uint32_t kTmemCols = 256;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
@@ -37,42 +49,47 @@ constexpr float kRescaleThreshold = 8.0f;  // log2 units
 template <int D>
 struct TcSmem {
   static constexpr int kHalves = D / 64;
-  static constexpr int kQBytes = kHalves * 128 * 128;         // 128 rows x D bf16
-  static constexpr int kTileBytes = kHalves * kTcTile * 128;  // 64 keys x D bf16 (K or V)
-  static constexpr int kStageBytes = 2 * kTileBytes;
-  static constexpr int kPBytes = 128 * 128;                   // 128 rows x 64 keys bf16
+  static constexpr int kStages = D == 128 ? 6 : 12;
+  static constexpr int kQBytes = kHalves * 128 * 128;                // 128 rows x D bf16
+  static constexpr int kPageBytes = kHalves * kPage * 128;           // V: [half][16 rows][128 B]
+  static constexpr int kTileBytes = (kTcTile / kPage) * kPageBytes;  // 64 keys x D bf16 (K or V)
   static constexpr int kQOff = 0;
-  static constexpr int kKVOff = kQOff + kQBytes;
-  static constexpr int kPOff = kKVOff + kTcStages * kStageBytes;
-  static constexpr int kBarOff = kPOff + 2 * kPBytes;
-  static constexpr int kBytes = kBarOff + 256;
+  static constexpr int kKOff = kQOff + kQBytes;
+  static constexpr int kVOff = kKOff + kStages * kTileBytes;
+  static constexpr int kBarOff = kVOff + kStages * kTileBytes;
+  static constexpr int kBytes = kBarOff + 512;
   static constexpr int kAlloc = kBytes + 1024;  // slack for 1024-byte alignment
 };
+constexpr int kTcStages = TcSmem<128>::kStages;
 
+// tm_k: 4-D {64 columns, 16 rows, heads, blocks}, one 64-column half of a
+// page per box; tm_v: 5-D {64 columns, 16 rows, halves, heads, blocks}, a
+// whole page per box.
 template <int D, int CAP>
 __global__ void __launch_bounds__(kTcThreads, 1)
 verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __grid_constant__ CUtensorMap tm_k,
                            const __grid_constant__ CUtensorMap tm_v) {
   using L = TcSmem<D>;
   constexpr int kHalves = L::kHalves;
+  constexpr int S = L::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = smem + L::kQOff;
-  uint8_t* sKV = smem + L::kKVOff;
-  uint8_t* sP = smem + L::kPOff;
+  uint8_t* sK = smem + L::kKOff;
+  uint8_t* sV = smem + L::kVOff;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::kBarOff);
-  uint64_t* kv_full = bars;                // [kTcStages]
-  uint64_t* kv_empty = bars + kTcStages;   // [kTcStages]
-  uint64_t* s_full = bars + 2 * kTcStages;  // [2]
-  uint64_t* s_empty = s_full + 2;           // [2]
-  uint64_t* p_full = s_empty + 2;           // [2]
-  uint64_t* pv_done = p_full + 2;           // [2]
+  uint64_t* k_full = bars;             // [S]
+  uint64_t* k_empty = bars + S;        // [S]
+  uint64_t* v_full = bars + 2 * S;     // [S]
+  uint64_t* v_empty = bars + 3 * S;    // [S]
+  uint64_t* s_full = bars + 4 * S;     // [2]
+  uint64_t* p_full = s_full + 2;       // [2]
+  uint64_t* pv_done = p_full + 2;      // [2]
   uint64_t* o_final = pv_done + 2;
   uint64_t* q_ready = o_final + 1;
-  uint64_t* mma_done = q_ready + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(q_ready + 1);
 
-  // ---- work item (same decode as the mma.sync kernel)
+  // ---- work item
   const int item = blockIdx.x;
   const int ui = find_user<CAP>(p.item_off, p.B, item);
   const AttnUser U = p.u[ui];
@@ -85,24 +102,24 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
   const int row0 = rb * 128;
   const int kv_begin = split * U.split_len;
   const int kv_end = min(kv_begin + U.split_len, U.kv_len);
-  const int ntiles = (kv_end - kv_begin + kTcTile - 1) / kTcTile;
+  const int ntiles = max(0, (kv_end - kv_begin + kTcTile - 1) / kTcTile);  // 0: an empty split
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kTcStages; ++s) {
-      mbar_init(&kv_full[s], 1);
-      mbar_init(&kv_empty[s], 1);
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
+      mbar_init(&v_full[s], 1);
+      mbar_init(&v_empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&s_full[b], 1);
-      mbar_init(&s_empty[b], 4);
       mbar_init(&p_full[b], 4);
       mbar_init(&pv_done[b], 1);
     }
     mbar_init(o_final, 1);
     mbar_init(q_ready, 4);
-    mbar_init(mma_done, 1);
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
@@ -118,6 +135,8 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const uint32_t tS0 = tmem, tO = tmem + 128;
+  float fin_m = -INFINITY, fin_l = 0.f;  // softmax threads: row state after the last tile
+  bool fin_ok = false;
   pdl_wait_prior_grid();
   pdl_launch_dependents();
 
@@ -132,93 +151,108 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
       const int page = page_base + group * 32 + lane;
       return page < n_pages ? __ldg(bt + page) : 0;
     };
+    constexpr int kPages = kTcTile / kPage;
+    constexpr int kKBoxes = kPages * kHalves;  // K boxes per tile; V: kPages
+    // lane -> its box: K (page, half) for lanes < kKBoxes, V page for the next kPages
+    const int kb = lane < kKBoxes ? lane : 0;
+    const int vb = lane - kKBoxes;
+    const int my_pg = lane < kKBoxes ? kb / kHalves : (vb & (kPages - 1));
+    const int my_hf = kb % kHalves;
     int cur = fetch(0);
     int nxt = fetch(1);
     int issued = 0;
     for (int j = 0; j < ntiles; ++j) {
-      const int st = j % kTcStages;
+      const int st = j % S;
       if ((j & 7) == 0 && j > 0) {
         cur = nxt;
         nxt = fetch((j >> 3) + 1);
       }
+      const int bk = __shfl_sync(0xffffffffu, cur, (j & 7) * kPages + my_pg);
+      const uint32_t ph = ((j / S) - 1) & 1;
+      const uint32_t koff = st * L::kTileBytes + my_hf * (kTcTile * 128) + my_pg * (kPage * 128);
+      const uint32_t voff = st * L::kTileBytes + my_pg * L::kPageBytes;
+      // K tile
       bool go = true;
-      if (j >= kTcStages && lane == 0) go = mbar_wait(&kv_empty[st], ((j / kTcStages) - 1) & 1, p.status);
-      go = __shfl_sync(0xffffffffu, go, 0);
-      if (!go) break;
-      int blk[kTcTile / kPage];
-#pragma unroll
-      for (int pg = 0; pg < kTcTile / kPage; ++pg) blk[pg] = __shfl_sync(0xffffffffu, cur, (j & 7) * 4 + pg);
-      // one box (one page, one 64-column half, K or V) per lane: a tile's
-      // boxes go out in a single warp-wide TMA instruction
-      if (lane == 0) mbar_arrive_expect_tx(&kv_full[st], L::kStageBytes);
+      if (j >= S && lane == 0) go = mbar_wait(&k_empty[st], ph, p.status);
+      if (!__shfl_sync(0xffffffffu, go, 0)) break;
+      if (lane == 0) mbar_arrive_expect_tx(&k_full[st], L::kTileBytes);
       __syncwarp();
-      {
-        constexpr int kBoxes = (kTcTile / kPage) * kHalves;  // per K tile (and per V tile)
-        if (lane < 2 * kBoxes) {
-          const int isv = lane >= kBoxes;
-          const int bx = isv ? lane - kBoxes : lane;
-          const int pg = bx / kHalves, hf = bx % kHalves;
-          int bk = blk[0];
-#pragma unroll
-          for (int q = 1; q < kTcTile / kPage; ++q)
-            if (pg == q) bk = blk[q];
-          uint8_t* dst = sKV + st * L::kStageBytes + (isv ? L::kTileBytes : 0) + hf * (kTcTile * 128) +
-                         pg * kPage * 128;
-          tma_load_4d(dst, isv ? &tm_v : &tm_k, hf * 64, 0, h, bk, &kv_full[st]);
-        }
-      }
+      if (lane < kKBoxes) tma_load_4d(sK + koff, &tm_k, my_hf * 64, 0, h, bk, &k_full[st]);
+      // V tile
+      if (j >= S && lane == 0) go = mbar_wait(&v_empty[st], ph, p.status);
+      if (!__shfl_sync(0xffffffffu, go, 0)) break;
+      if (lane == 0) mbar_arrive_expect_tx(&v_full[st], L::kTileBytes);
+      __syncwarp();
+      if (lane >= kKBoxes && lane < kKBoxes + kPages) tma_load_5d(sV + voff, &tm_v, 0, 0, 0, h, bk, &v_full[st]);
       ++issued;
     }
+    // copies still in flight must land before the CTA can exit
     if (lane == 0)
-      for (int j = max(0, issued - kTcStages); j < issued; ++j)
-        mbar_wait(&kv_full[j % kTcStages], (j / kTcStages) & 1, p.status);
+      for (int j = max(0, issued - S); j < issued; ++j) {
+        mbar_wait(&k_full[j % S], (j / S) & 1, p.status);
+        mbar_wait(&v_full[j % S], (j / S) & 1, p.status);
+      }
   } else if (warp == 1) {
     // ----------------------------------------------------- MMA issuer (1 thread)
     if (lane == 0) {
       constexpr uint32_t kIdQK = idesc_bf16_f32(128, kTcTile, false, false);
-      constexpr uint32_t kIdPV = idesc_bf16_f32(128, 64, false, true);
       const uint32_t q_addr = smem_addr(sQ);
-      const uint32_t kv_addr = smem_addr(sKV);
-      const uint32_t p_addr = smem_addr(sP);
+      constexpr uint32_t kIdPV = idesc_bf16_f32(128, 64, false, true);
+      const uint32_t k_addr = smem_addr(sK);
+      const uint32_t v_addr = smem_addr(sV);
       bool ok = mbar_wait(q_ready, 0, p.status);
-      auto issue_pv = [&](int jj) -> bool {
-        const int st = jj % kTcStages, b = jj & 1;
-        if (!mbar_wait(&p_full[b], (jj >> 1) & 1, p.status)) return false;
-        tc_fence_after();
-        const uint32_t v_addr = kv_addr + st * L::kStageBytes + L::kTileBytes;
+      int jq = 0, jp = 0;  // next Q K^T, next P V
+      uint64_t idle_since = 0;
+      while (ok && jp < ntiles) {
+        bool did = false;
+        // S[jq & 1] is free once P V of tile jq - 2 has been issued (the
+        // tensor core runs one thread's MMAs in issue order)
+        if (jq < ntiles && jp >= jq - 1 && mbar_try_wait(&k_full[jq % S], (jq / S) & 1)) {
+          tc_fence_after();
+          const uint32_t kt = k_addr + (jq % S) * L::kTileBytes;
 #pragma unroll
-        for (int hf = 0; hf < kHalves; ++hf) {
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t hoff = (kk >> 2) * (128 * 128), koff = (kk >> 2) * (kTcTile * 128);
+            const uint64_t a = smem_desc_sw128(q_addr + hoff + (kk & 3) * 32, 0, 1024);
+            const uint64_t bd = smem_desc_sw128(kt + koff + (kk & 3) * 32, 0, 1024);
+            tc_mma(tS0 + (jq & 1) * kTcTile, a, bd, kIdQK, kk > 0 ? 1u : 0u);
+          }
+          tc_commit(&s_full[jq & 1]);
+          tc_commit(&k_empty[jq % S]);
+          ++jq;
+          did = true;
+        }
+        if (jp < jq && mbar_try_wait(&p_full[jp & 1], (jp >> 1) & 1) &&
+            mbar_try_wait(&v_full[jp % S], (jp / S) & 1)) {
+          tc_fence_after();
+          const uint32_t vt = v_addr + (jp % S) * L::kTileBytes;
+          const uint32_t pt = tS0 + (jp & 1) * kTcTile;  // P: 32 columns of bf16 pairs
 #pragma unroll
-          for (int kk = 0; kk < kTcTile / 16; ++kk) {
-            const uint64_t a = smem_desc_sw128(p_addr + b * L::kPBytes + kk * 32, 0, 1024);
-            const uint64_t bd = smem_desc_sw128(v_addr + hf * (kTcTile * 128) + kk * 16 * 128, 1024, 1024);
-            tc_mma(tO + hf * 64, a, bd, kIdPV, (jj > 0 || kk > 0) ? 1u : 0u);
+          for (int hf = 0; hf < kHalves; ++hf) {
+#pragma unroll
+            for (int kk = 0; kk < kTcTile / 16; ++kk) {
+              const uint64_t bd = smem_desc_sw128(vt + kk * L::kPageBytes + hf * (kPage * 128), 1024, 1024);
+              tc_mma_ts(tO + hf * 64, pt + kk * 8, bd, kIdPV, (jp > 0 || kk > 0) ? 1u : 0u);
+            }
+          }
+          tc_commit(&pv_done[jp & 1]);
+          tc_commit(&v_empty[jp % S]);
+          ++jp;
+          did = true;
+        }
+        if (did) {
+          idle_since = 0;
+        } else {
+          const uint64_t now = global_timer_ns();
+          if (idle_since == 0) {
+            idle_since = now;
+          } else if (now - idle_since > kWaitLimitNs) {
+            atomicOr(p.status, kDevErrWaitTimeout);
+            ok = false;
           }
         }
-        tc_commit(&pv_done[b]);
-        tc_commit(&kv_empty[st]);
-        return true;
-      };
-      for (int j = 0; ok && j < ntiles; ++j) {
-        const int st = j % kTcStages, b = j & 1;
-        if (!mbar_wait(&kv_full[st], (j / kTcStages) & 1, p.status)) { ok = false; break; }
-        if (j >= 2 && !mbar_wait(&s_empty[b], ((j - 2) >> 1) & 1, p.status)) { ok = false; break; }
-        tc_fence_after();
-        const uint32_t k_addr = kv_addr + st * L::kStageBytes;
-#pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t hoff = (kk >> 2) * (128 * 128), koff = (kk >> 2) * (kTcTile * 128);
-          const uint64_t a = smem_desc_sw128(q_addr + hoff + (kk & 3) * 32, 0, 1024);
-          const uint64_t bd = smem_desc_sw128(k_addr + koff + (kk & 3) * 32, 0, 1024);
-          tc_mma(tS0 + b * kTcTile, a, bd, kIdQK, kk > 0 ? 1u : 0u);
-        }
-        tc_commit(&s_full[b]);
-        if (j >= 1 && !issue_pv(j - 1)) { ok = false; break; }
       }
-      if (ok && ntiles > 0) ok = issue_pv(ntiles - 1);
       tc_commit(o_final);
-      tc_commit(mma_done);
-      mbar_wait(mma_done, 0, p.status);
     }
   } else {
     // ----------------------------------------- softmax / epilogue (row per thread)
@@ -245,27 +279,25 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
     }
 
     const int last_vis = U.ctx + t;  // last visible key of this row
-    // warps whose 32 rows are all padding only keep the barrier phases in step
+    // warps whose 32 rows are all padding write zero P, so every lane of P
+    // the tensor core reads is defined
     const bool active = row0 + quad * 32 < M;
     const float sl2 = p.scale_log2;
     float m = -INFINITY, l = 0.f;
     bool ok = true;
     for (int j = 0; j < ntiles; ++j) {
-      const int b = j & 1, st = j % kTcStages;
+      const int b = j & 1, st = j % S;
       const int key0 = kv_begin + j * kTcTile;
       ok = __all_sync(0xffffffffu, mbar_wait(&s_full[b], (j >> 1) & 1, p.status));
       if (!ok) break;
-      uint32_t sr[2][32];
+      tc_fence_after();
+      uint32_t pk[kTcTile / 2];
+#pragma unroll
+      for (int c = 0; c < kTcTile / 2; ++c) pk[c] = 0u;
       if (active) {
-        tc_fence_after();
+        uint32_t sr[2][32];
         tmem_ld32(tS0 + b * kTcTile + lane_base, sr[0]);
         tmem_ld32(tS0 + b * kTcTile + 32 + lane_base, sr[1]);
-        tc_fence_before();
-      }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&s_empty[b]);
-
-      if (active) {
         // raw scores; the causal rule key <= C_i + t only bites near the end
         float s[kTcTile];
         float mr = -INFINITY;
@@ -286,6 +318,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
           m = mt;
         }
         if (j > 0 && __any_sync(0xffffffffu, grow && factor != 1.f)) {
+          // every earlier P V has to be done before O is touched
           ok = __all_sync(0xffffffffu, mbar_wait(&pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1, p.status));
           if (!ok) break;
           tc_fence_after();
@@ -297,11 +330,9 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
             for (int k = 0; k < 32; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * factor);
             tmem_st32(tO + cc * 32 + lane_base, o);
           }
-          tc_fence_before();
         }
         l *= factor;
         const float nb = m == -INFINITY ? 0.f : -m;
-        uint32_t pk[kTcTile / 2];
 #pragma unroll
         for (int c = 0; c < kTcTile; c += 2) {
           const float p0 = fast_exp2(__fmaf_rn(s[c], sl2, nb));
@@ -309,39 +340,36 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
           l += p0 + p1;
           pk[c >> 1] = pack_bf16x2(p0, p1);
         }
-        // P buffer b was last read by the PV of tile j-2
-        if (j >= 2) {
-          ok = __all_sync(0xffffffffu, mbar_wait(&pv_done[b], ((j - 2) >> 1) & 1, p.status));
-          if (!ok) break;
-        }
-        uint8_t* prow = sP + b * L::kPBytes + r * 128;
-#pragma unroll
-        for (int ch = 0; ch < 8; ++ch)
-          *reinterpret_cast<uint4*>(prow + ((ch ^ (r & 7)) << 4)) =
-              make_uint4(pk[4 * ch], pk[4 * ch + 1], pk[4 * ch + 2], pk[4 * ch + 3]);
       }
+      // P over the first 32 columns of S[b] (already read); the P V that
+      // read this buffer two tiles ago completed before S[b] was written
+      tmem_st32(tS0 + b * kTcTile + lane_base, pk);
       // V rows past kv_len may hold anything; zero them before P V reads them
       if (key0 + kTcTile > U.kv_len) {
-        ok = __all_sync(0xffffffffu, mbar_wait(&kv_full[st], (j / kTcStages) & 1, p.status));
+        ok = __all_sync(0xffffffffu, mbar_wait(&v_full[st], (j / S) & 1, p.status));
         if (!ok) break;
-        uint8_t* vt = sKV + st * L::kStageBytes + L::kTileBytes;
+        uint8_t* vt = sV + st * L::kTileBytes;
         const int first = U.kv_len - key0;  // first key row to clear
         const int nchunks = (kTcTile - first) * kHalves * 8;
         for (int c = threadIdx.x - 64; c < nchunks; c += 128) {
           const int row = first + c / (kHalves * 8);
-          const int rem = c % (kHalves * 8);
-          *reinterpret_cast<uint4*>(vt + (rem >> 3) * (kTcTile * 128) + row * 128 + ((rem & 7) << 4)) =
-              make_uint4(0, 0, 0, 0);
+          const int rem = c % (kHalves * 8);  // every 16-byte chunk of the row, in any order
+          *reinterpret_cast<uint4*>(vt + (row / kPage) * L::kPageBytes + (rem >> 3) * (kPage * 128) +
+                                    (row % kPage) * 128 + ((rem & 7) << 4)) = make_uint4(0, 0, 0, 0);
         }
+        fence_proxy_async_smem();
       }
-      fence_proxy_async_smem();
+      tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&p_full[b]);
     }
 
     // ---- epilogue: O row from TMEM
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(o_final, 0, p.status));
-    if (ok && active) {
+    fin_m = m;
+    fin_l = l;
+    fin_ok = ok;
+    if (ok && active && p.cluster <= 1) {
       tc_fence_after();
       const float inv = l > 0.f ? 1.f / l : 0.f;
       __nv_bfloat16* orow = p.out + (static_cast<size_t>(U.q_off + t) * p.Hq + h * p.G + g) * D;
@@ -368,8 +396,91 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
         }
       }
       if (valid && U.nsplit > 1) p.part_ml[prow_idx] = make_float2(m, l);
-      tc_fence_before();
     }
+    tc_fence_before();
+  }
+
+  if (p.cluster > 1) {
+    // ---- split merge inside the cluster (every thread takes both barriers)
+    constexpr int kSlot = 128 * 8 + 128 * D * 4;  // (m, l) per row, then O as [D/4][128] float4
+    const uint32_t crank = cluster_ctarank();
+    const int quad = warp & 3;
+    const int r = quad * 32 + lane;
+    const int rg = row0 + r;
+    const bool valid = rg < M;
+    const bool active = warp >= 2 && row0 + quad * 32 < M;
+    const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;
+    uint8_t* xbuf = sK;  // rank 0's rings, drained once every rank is here
+    cluster_arrive_release();
+    cluster_wait_acquire();
+    if (active && crank > 0 && fin_ok) {
+      const uint32_t slot = dsmem_map(xbuf + (crank - 1) * kSlot, 0);
+      if (valid) dsmem_st_f32x2(slot + r * 8, fin_m, fin_l);
+      tc_fence_after();
+#pragma unroll 1
+      for (int cc = 0; cc < D / 32; ++cc) {
+        uint32_t o[32];
+        tmem_ld32(tO + cc * 32 + lane_base, o);
+        if (valid && fin_l > 0.f) {
+#pragma unroll
+          for (int k = 0; k < 8; ++k)
+            dsmem_st_f32x4(slot + 1024 + ((cc * 8 + k) * 128 + r) * 16, __uint_as_float(o[4 * k]),
+                           __uint_as_float(o[4 * k + 1]), __uint_as_float(o[4 * k + 2]),
+                           __uint_as_float(o[4 * k + 3]));
+        }
+      }
+    }
+    cluster_arrive_release();
+    cluster_wait_acquire();
+    if (active && crank == 0 && fin_ok) {
+      const int C = p.cluster;
+      const int t = rg / p.G, g = rg % p.G;
+      float mx = fin_m;
+      for (int s = 1; s < C; ++s)
+        mx = fmaxf(mx, reinterpret_cast<const float2*>(xbuf + (s - 1) * kSlot)[r].x);
+      // weights 2^(m_s - mx) (log2 units); an empty split weighs 0
+      const float w0 = fin_m == -INFINITY ? 0.f : fast_exp2(fin_m - mx);
+      float l = w0 * fin_l;
+      for (int s = 1; s < C; ++s) {
+        const float2 ml = reinterpret_cast<const float2*>(xbuf + (s - 1) * kSlot)[r];
+        l += ml.x == -INFINITY ? 0.f : fast_exp2(ml.x - mx) * ml.y;
+      }
+      const float inv = l > 0.f ? 1.f / l : 0.f;
+      __nv_bfloat16* orow = p.out + (static_cast<size_t>(U.q_off + t) * p.Hq + h * p.G + g) * D;
+      tc_fence_after();
+#pragma unroll 1
+      for (int cc = 0; cc < D / 32; ++cc) {
+        uint32_t o[32];
+        tmem_ld32(tO + cc * 32 + lane_base, o);
+        float acc[32];
+#pragma unroll
+        for (int k = 0; k < 32; ++k) acc[k] = w0 > 0.f ? w0 * __uint_as_float(o[k]) : 0.f;
+        for (int s = 1; s < C; ++s) {
+          const float2 ml = reinterpret_cast<const float2*>(xbuf + (s - 1) * kSlot)[r];
+          if (!(ml.x > -INFINITY) || !(ml.y > 0.f)) continue;
+          const float w = fast_exp2(ml.x - mx);
+          const float4* os = reinterpret_cast<const float4*>(xbuf + (s - 1) * kSlot + 1024);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const float4 v = os[(cc * 8 + k) * 128 + r];
+            acc[4 * k] += w * v.x;
+            acc[4 * k + 1] += w * v.y;
+            acc[4 * k + 2] += w * v.z;
+            acc[4 * k + 3] += w * v.w;
+          }
+        }
+        if (valid) {
+          uint4* dst = reinterpret_cast<uint4*>(orow + cc * 32);
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            dst[k] = make_uint4(pack_bf16x2(acc[8 * k] * inv, acc[8 * k + 1] * inv),
+                                pack_bf16x2(acc[8 * k + 2] * inv, acc[8 * k + 3] * inv),
+                                pack_bf16x2(acc[8 * k + 4] * inv, acc[8 * k + 5] * inv),
+                                pack_bf16x2(acc[8 * k + 6] * inv, acc[8 * k + 7] * inv));
+        }
+      }
+    }
+    tc_fence_before();
   }
 
   __syncthreads();

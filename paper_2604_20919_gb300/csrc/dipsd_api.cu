@@ -66,18 +66,30 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
   return fn;
 }
 
-// Paged cache [num_blocks][Hkv][16][D] bf16 as a 4-D tensor (D innermost);
-// one box = one page of one head, 64 columns wide, 128-byte swizzle.
-bool encode_cache_map(CUtensorMap* map, const void* base, int num_blocks, int Hkv, int D) {
+// Paged cache [num_blocks][Hkv][16][D] bf16 as tensor maps with the 128-byte
+// swizzle.  K (4-D: D columns, 16 rows, heads, blocks): one box = one
+// 64-column half of one page of one head.  V (5-D: 64 columns, 16 rows of
+// 2*D bytes, D/64 halves 128 bytes apart, heads, blocks): one box = a whole
+// page of one head, stored half after half.
+bool encode_cache_map(CUtensorMap* map, const void* base, int num_blocks, int Hkv, int D, bool whole_page) {
   auto enc = tensor_map_encoder();
   if (!enc) return false;
-  cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)kPage, (cuuint64_t)Hkv, (cuuint64_t)num_blocks};
-  cuuint64_t strides[3] = {(cuuint64_t)D * 2, (cuuint64_t)kPage * D * 2, (cuuint64_t)Hkv * kPage * D * 2};
-  cuuint32_t box[4] = {64, (cuuint32_t)kPage, 1, 1};
-  cuuint32_t estr[4] = {1, 1, 1, 1};
-  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, estr,
-             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  const cuuint64_t row = static_cast<cuuint64_t>(D) * 2;
+  cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+  if (!whole_page) {
+    cuuint64_t dims[4] = {(cuuint64_t)D, (cuuint64_t)kPage, (cuuint64_t)Hkv, (cuuint64_t)num_blocks};
+    cuuint64_t strides[3] = {row, kPage * row, (cuuint64_t)Hkv * kPage * row};
+    cuuint32_t box[4] = {64, (cuuint32_t)kPage, 1, 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  }
+  cuuint64_t dims[5] = {64, (cuuint64_t)kPage, (cuuint64_t)(D / 64), (cuuint64_t)Hkv, (cuuint64_t)num_blocks};
+  cuuint64_t strides[4] = {row, 128, kPage * row, (cuuint64_t)Hkv * kPage * row};
+  cuuint32_t box[5] = {64, (cuuint32_t)kPage, (cuuint32_t)(D / 64), 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 // --------------------------------------------------------------- launching
@@ -129,6 +141,7 @@ struct AttnPlan {
   int B = 0, Hq = 0, Hkv = 0, G = 0, D = 0;
   int NW = 4, stages = 3;
   int n_items = 0, n_merge = 0;
+  int cluster = 0;  // > 1: splits merged inside a thread-block cluster of this size
   long long part_rows = 0;
   std::vector<AttnUser> u;
   std::vector<int> item_off, merge_off;
@@ -172,15 +185,20 @@ void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int
   const int rows_cta = 128;
   const int slots = sms;
 
-  int forced = 0;
+  int forced = 0, forced_cluster = 0;
   if (const char* e = std::getenv("DIPSD_ATTN_SPLIT_TILES")) forced = std::atoi(e);
+  if (const char* e = std::getenv("DIPSD_ATTN_CLUSTER")) forced_cluster = std::atoi(e);
   const int cands[] = {1, 2, 3, 4, 5, 6, 8, 10, 12, 16, 20, 24, 32, 40, 48, 64, 96, 128, 192, 256, 384, 512, 1 << 30};
+  // Costs in tile units: an item pays its tiles plus ~2 of prologue and
+  // epilogue; splits merged by the separate merge kernel pay ~3 more (its
+  // launch behind the attention grid), splits merged in a cluster ~0.5.
   double best = 1e300;
   int best_c = 1 << 30;
   for (int c : cands) {
     if (forced > 0) c = forced;
     double total = 0, max_item = 0;
     long long items = 0;
+    bool any_split = false;
     for (int i = 0; i < B; ++i) {
       const int tiles = (ctx[i] + L[i] + 1 + kAttnTile - 1) / kAttnTile;
       const int cc = std::max(1, std::min(c, tiles));
@@ -192,15 +210,38 @@ void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int
       total += item * ns * rb * Hkv;
       items += static_cast<long long>(ns) * rb * Hkv;
       max_item = std::max(max_item, item);
+      any_split = any_split || ns > 1;
     }
     if (items > (1ll << 30)) continue;
     // items are near-uniform (one split length): waves x longest item, but
     // never better than perfect balance plus one item
     const double waves = std::ceil(static_cast<double>(items) / slots);
-    const double cost = std::max(waves * max_item, total / slots + 0.5 * max_item);
+    const double cost = std::max(waves * max_item, total / slots + 0.5 * max_item) + (any_split ? 3.0 : 0.0);
     if (cost < best - 1e-9) { best = cost; best_c = c; }
     if (forced > 0) break;
   }
+
+  // Cluster merge: every user's KV in the same number C of splits (one wave,
+  // the exchange buffer of C - 1 ranks fitting rank 0's rings).
+  const int max_cluster = D == 128 ? 3 : 6;
+  int best_cl = 0;
+  double best_b = 1e300;
+  for (int C = 2; C <= max_cluster && forced == 0; ++C) {
+    if (forced_cluster > 0) C = std::min(forced_cluster, max_cluster);
+    long long items = 0;
+    double max_item = 0;
+    for (int i = 0; i < B; ++i) {
+      const int tiles = (ctx[i] + L[i] + 1 + kAttnTile - 1) / kAttnTile;
+      const int rb = (pl.G * (L[i] + 1) + rows_cta - 1) / rows_cta;
+      items += static_cast<long long>(C) * rb * Hkv;
+      max_item = std::max(max_item, (tiles + C - 1) / C + 2.5);
+    }
+    if (items <= slots || forced_cluster > 0) {
+      if (max_item < best_b) { best_b = max_item; best_cl = C; }
+    }
+    if (forced_cluster > 0) break;
+  }
+  pl.cluster = (forced_cluster > 0 || best_b < best) && best_cl > 1 ? best_cl : 0;
 
   pl.u.assign(B, AttnUser{});
   pl.item_off.assign(B + 1, 0);
@@ -215,17 +256,23 @@ void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int
     U.kv_len = ctx[i] + U.T;
     U.bt_row = bt_rows ? bt_rows[i] : i;
     const int tiles = (U.kv_len + kAttnTile - 1) / kAttnTile;
-    const int cc = std::max(1, std::min(best_c, tiles));
-    int ns = (tiles + cc - 1) / cc;
-    const int st = (tiles + ns - 1) / ns;
-    ns = (tiles + st - 1) / st;
+    int ns, st;
+    if (pl.cluster > 1) {
+      ns = pl.cluster;  // trailing splits may be empty when tiles < C
+      st = (tiles + ns - 1) / ns;
+    } else {
+      const int cc = std::max(1, std::min(best_c, tiles));
+      ns = (tiles + cc - 1) / cc;
+      st = (tiles + ns - 1) / ns;
+      ns = (tiles + st - 1) / st;
+    }
     U.nsplit = ns;
     U.split_len = st * kAttnTile;
     U.n_rb = (pl.G * U.T + rows_cta - 1) / rows_cta;
     pl.item_off[i] = static_cast<int>(items);
     pl.merge_off[i] = static_cast<int>(merge);
     items += static_cast<long long>(ns) * U.n_rb * Hkv;
-    if (ns > 1) {
+    if (ns > 1 && pl.cluster <= 1) {
       pl.part_off[i] = part;
       part += static_cast<long long>(ns) * Hkv * pl.G * U.T;
       merge += static_cast<long long>(U.T) * Hq;
@@ -249,6 +296,7 @@ void fill_attn_params(AttnParams<CAP>& p, const AttnPlan& pl, const void* q, voi
   p.part_ml = reinterpret_cast<float2*>(region);
   p.part_o = reinterpret_cast<float*>(region + align_up(pl.part_rows * sizeof(float2), 256));
   p.status = status;
+  p.cluster = pl.cluster;
   p.B = pl.B; p.Hq = pl.Hq; p.Hkv = pl.Hkv; p.G = pl.G; p.max_blocks = max_blocks;
   p.n_items = pl.n_items; p.n_merge = pl.n_merge;
   p.scale_log2 = scale * 1.4426950408889634f;
@@ -266,7 +314,8 @@ int launch_attention_tc_t(const AttnPlan& pl, const AttnParams<CAP>& p, const CU
     std::lock_guard<std::mutex> lock(mu);
     if (!allow_smem(kern, TcSmem<D>::kAlloc, attr_done)) return DIPSD_ERR_CUDA;
   }
-  if (launch(kern, dim3(pl.n_items), dim3(kTcThreads), TcSmem<D>::kAlloc, s, 0, pdl, p, tk, tv) != cudaSuccess)
+  if (launch(kern, dim3(pl.n_items), dim3(kTcThreads), TcSmem<D>::kAlloc, s, pl.cluster > 1 ? pl.cluster : 0, pdl,
+             p, tk, tv) != cudaSuccess)
     return DIPSD_ERR_CUDA;
   if (pl.n_merge > 0) {
     auto mk = verify_attention_merge_kernel<D, CAP>;
@@ -283,8 +332,8 @@ int run_attention_cap(const AttnPlan& pl, const void* q, const void* kc, const v
   static thread_local AttnParams<CAP> p;
   fill_attn_params<CAP>(p, pl, q, out, bt, max_blocks, scale, status, region);
   alignas(64) CUtensorMap tk, tv;
-  if (!encode_cache_map(&tk, kc, num_blocks, pl.Hkv, pl.D) ||
-      !encode_cache_map(&tv, vc, num_blocks, pl.Hkv, pl.D))
+  if (!encode_cache_map(&tk, kc, num_blocks, pl.Hkv, pl.D, false) ||
+      !encode_cache_map(&tv, vc, num_blocks, pl.Hkv, pl.D, true))
     return DIPSD_ERR_CUDA;
   return pl.D == 128 ? launch_attention_tc_t<128, CAP>(pl, p, tk, tv, s, pdl)
                      : launch_attention_tc_t<64, CAP>(pl, p, tk, tv, s, pdl);

@@ -75,6 +75,24 @@ def test_attention_forced_splits(cuda_lib, split_tiles):
     check_attention(out, _full_reference(b))
 
 
+@pytest.mark.parametrize("cluster,D", [("2", 128), ("3", 128), ("6", 64)])
+def test_attention_cluster_merge(cuda_lib, cluster, D):
+    """KV splits merged inside a thread-block cluster, including empty splits
+    (a user with fewer 64-key tiles than splits)."""
+    b = make_batch([5, 0, 8, 2, 1], [1500, 3000, 333, 64, 0], Hq=64 if D == 128 else 16, Hkv=8 if D == 128 else 2,
+                   D=D, V=64, seed=23)
+    old = os.environ.get("DIPSD_ATTN_CLUSTER")
+    os.environ["DIPSD_ATTN_CLUSTER"] = cluster
+    try:
+        out = _run(cuda_lib, b)
+    finally:
+        if old is None:
+            del os.environ["DIPSD_ATTN_CLUSTER"]
+        else:
+            os.environ["DIPSD_ATTN_CLUSTER"] = old
+    check_attention(out, _full_reference(b))
+
+
 def test_attention_ignores_slots_past_kv_len(cuda_lib):
     """NaN in cache slots past each user's kv_len and in unused pages never reaches the output."""
     b = make_batch([2, 5, 0], [30, 500, 1], Hq=64, Hkv=8, D=128, V=64, seed=22)
