@@ -18,10 +18,11 @@
 //               group ahead.
 //   warp 1      allocates TMEM; one thread issues tcgen05.mma as operands
 //               become ready (no fixed order between the two products):
-//                 S[b] = Q K^T      (A = Q from shared memory, M=128, N=64)
+//                 S[b] = Q K^T      (A = Q from tensor memory, M=128, N=64)
 //                 O   += P[b] V     (A = P from tensor memory; a 16-key step
 //                                    is one page of V; two N=64 halves)
-//   warps 2..5  one query row per thread (TMEM lane = row): load S[b] with
+//   warps 2..5  one query row per thread (TMEM lane = row): put the Q row
+//               in TMEM, then per tile load S[b] with
 //               tcgen05.ld, causal mask, online softmax in log2 units with a
 //               lazy rescale (O in TMEM is rescaled only when a row maximum
 //               grows by more than 2^8), write P as bf16 pairs into the first
@@ -31,9 +32,10 @@
 // block and head run as one thread-block cluster: the other ranks push their
 // rows into rank 0's drained rings through distributed shared memory and
 // rank 0 merges them with its own O straight from TMEM.
-// TMEM columns: S/P double buffer [0,64) [64,128), O [128, 128+D).  Shared
-// memory holds Q and the two rings (P never leaves tensor memory), which is
-// what leaves room for kStages tiles of K and of V in flight.
+// TMEM columns: S/P double buffer [0,64) [64,128), O [128, 128+D), Q [256,
+// 256 + D/2).  Shared memory holds only the two rings (Q and P live in
+// tensor memory, so no product re-reads an operand from shared memory every
+// tile), which leaves room for kStages tiles of K and of V in flight.
 #pragma once
 
 #include "attention.cuh"
@@ -43,18 +45,16 @@ namespace dipsd {
 
 constexpr int kTcThreads = 192;
 constexpr int kTcTile = 64;                // keys per tile
-constexpr uint32_t kTmemCols = 256;
+constexpr uint32_t kTmemCols = 512;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 
 template <int D>
 struct TcSmem {
   static constexpr int kHalves = D / 64;
-  static constexpr int kStages = D == 128 ? 6 : 12;
-  static constexpr int kQBytes = kHalves * 128 * 128;                // 128 rows x D bf16
+  static constexpr int kStages = D == 128 ? 7 : 12;
   static constexpr int kPageBytes = kHalves * kPage * 128;           // V: [half][16 rows][128 B]
   static constexpr int kTileBytes = (kTcTile / kPage) * kPageBytes;  // 64 keys x D bf16 (K or V)
-  static constexpr int kQOff = 0;
-  static constexpr int kKOff = kQOff + kQBytes;
+  static constexpr int kKOff = 0;
   static constexpr int kVOff = kKOff + kStages * kTileBytes;
   static constexpr int kBarOff = kVOff + kStages * kTileBytes;
   static constexpr int kBytes = kBarOff + 512;
@@ -74,7 +74,6 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
   constexpr int S = L::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* sQ = smem + L::kQOff;
   uint8_t* sK = smem + L::kKOff;
   uint8_t* sV = smem + L::kVOff;
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::kBarOff);
@@ -134,7 +133,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t tS0 = tmem, tO = tmem + 128;
+  const uint32_t tS0 = tmem, tO = tmem + 128, tQ = tmem + 256;
   float fin_m = -INFINITY, fin_l = 0.f;  // softmax threads: row state after the last tile
   bool fin_ok = false;
   pdl_wait_prior_grid();
@@ -196,7 +195,6 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
     // ----------------------------------------------------- MMA issuer (1 thread)
     if (lane == 0) {
       constexpr uint32_t kIdQK = idesc_bf16_f32(128, kTcTile, false, false);
-      const uint32_t q_addr = smem_addr(sQ);
       constexpr uint32_t kIdPV = idesc_bf16_f32(128, 64, false, true);
       const uint32_t k_addr = smem_addr(sK);
       const uint32_t v_addr = smem_addr(sV);
@@ -207,23 +205,21 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
         bool did = false;
         // S[jq & 1] is free once P V of tile jq - 2 has been issued (the
         // tensor core runs one thread's MMAs in issue order)
-        if (jq < ntiles && jp >= jq - 1 && mbar_try_wait(&k_full[jq % S], (jq / S) & 1)) {
+        if (jq < ntiles && jp >= jq - 1 && mbar_test_wait(&k_full[jq % S], (jq / S) & 1)) {
           tc_fence_after();
           const uint32_t kt = k_addr + (jq % S) * L::kTileBytes;
 #pragma unroll
           for (int kk = 0; kk < D / 16; ++kk) {
-            const uint32_t hoff = (kk >> 2) * (128 * 128), koff = (kk >> 2) * (kTcTile * 128);
-            const uint64_t a = smem_desc_sw128(q_addr + hoff + (kk & 3) * 32, 0, 1024);
-            const uint64_t bd = smem_desc_sw128(kt + koff + (kk & 3) * 32, 0, 1024);
-            tc_mma(tS0 + (jq & 1) * kTcTile, a, bd, kIdQK, kk > 0 ? 1u : 0u);
+            const uint64_t bd = smem_desc_sw128(kt + (kk >> 2) * (kTcTile * 128) + (kk & 3) * 32, 0, 1024);
+            tc_mma_ts(tS0 + (jq & 1) * kTcTile, tQ + kk * 8, bd, kIdQK, kk > 0 ? 1u : 0u);
           }
           tc_commit(&s_full[jq & 1]);
           tc_commit(&k_empty[jq % S]);
           ++jq;
           did = true;
         }
-        if (jp < jq && mbar_try_wait(&p_full[jp & 1], (jp >> 1) & 1) &&
-            mbar_try_wait(&v_full[jp % S], (jp / S) & 1)) {
+        if (jp < jq && mbar_test_wait(&p_full[jp & 1], (jp >> 1) & 1) &&
+            mbar_test_wait(&v_full[jp % S], (jp / S) & 1)) {
           tc_fence_after();
           const uint32_t vt = v_addr + (jp % S) * L::kTileBytes;
           const uint32_t pt = tS0 + (jp & 1) * kTcTile;  // P: 32 columns of bf16 pairs
@@ -263,17 +259,26 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
     const int t = rg / p.G, g = rg % p.G;
     const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;
 
-    // Q row -> shared memory (K-major, 128-byte swizzle); padding rows are zero
+    // Q row -> TMEM lane r as bf16 pairs (column c holds elements 2c, 2c+1);
+    // padding rows are zero
     {
-      const __nv_bfloat16* qrow = p.q + (static_cast<size_t>(U.q_off + t) * p.Hq + h * p.G + g) * D;
+      const uint4* qrow =
+          reinterpret_cast<const uint4*>(p.q + (static_cast<size_t>(U.q_off + t) * p.Hq + h * p.G + g) * D);
 #pragma unroll
-      for (int c = 0; c < D / 8; ++c) {
-        uint4 v = make_uint4(0, 0, 0, 0);
-        if (valid) v = __ldg(reinterpret_cast<const uint4*>(qrow) + c);
-        const int hf = c >> 3, ch = c & 7;
-        *reinterpret_cast<uint4*>(sQ + hf * (128 * 128) + r * 128 + ((ch ^ (r & 7)) << 4)) = v;
+      for (int cc = 0; cc < D / 64; ++cc) {
+        uint32_t w[32];
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          uint4 v = make_uint4(0, 0, 0, 0);
+          if (valid) v = __ldg(qrow + cc * 8 + c);
+          w[4 * c] = v.x;
+          w[4 * c + 1] = v.y;
+          w[4 * c + 2] = v.z;
+          w[4 * c + 3] = v.w;
+        }
+        tmem_st32(tQ + cc * 32 + lane_base, w);
       }
-      fence_proxy_async_smem();
+      tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(q_ready);
     }
