@@ -261,6 +261,19 @@ def run_dipsd(args):
         c = copies[k % R]
         dipsd.dipsd_spec_verify(b.L, c["z"], c["w"], c["d"], c["u"], outputs=outs, ws=ws)
 
+    # the verify tokens' own K/V rows (already in the cache), for the append path
+    bt_h = b.block_table.numpy()
+    pos = [(i, int(b.ctx[i]) + t) for i in range(b.B) for t in range(int(b.L[i]) + 1)]
+    blk = torch.tensor([int(bt_h[i, p // 16]) for i, p in pos], device=dev)
+    slot = torch.tensor([p % 16 for _, p in pos], device=dev)
+    new_k = b.k_cache[blk, :, slot].contiguous()
+    new_v = b.v_cache[blk, :, slot].contiguous()
+
+    def attn_append(k):
+        c = copies[k % R]
+        dipsd.dipsd_verify_attention_append(b.L, b.ctx, c["q"], new_k, new_v, c["kc"], c["vc"], bt, b.scale,
+                                            out=attn_out, ws=ws)
+
     def graph_of(fn, n):
         """A CUDA graph of n consecutive calls cycling over the R input copies,
         and the number of library kernels it launches per replay."""
@@ -317,12 +330,14 @@ def run_dipsd(args):
     g_step, launches = graph_of(step, n_steps)
     g_attn, _ = graph_of(attn_only, n_steps)
     g_spec, _ = graph_of(spec_only, n_steps)
+    g_app, _ = graph_of(attn_append, n_steps)
 
     sampler = ClockSampler(local)
     sampler.start()
     ms_step = timed(g_step, n_steps)
     ms_attn = timed(g_attn, n_steps)
     ms_spec = timed(g_spec, n_steps)
+    ms_app = timed(g_app, n_steps)
     lat_step = cold_latency(step, min(args.steps, 50))
 
     # end to end through the same call: every step copies its inputs from pinned
@@ -399,6 +414,8 @@ def run_dipsd(args):
         "spec_verify": {"ms": ms_spec, "alg_bytes": s_bytes, "gbs": s_bytes / ms_spec / 1e6,
                         "frac_of_measured_hbm": s_bytes / ms_spec / 1e6 / hbm_peak,
                         "frac_of_8000": s_bytes / ms_spec / 1e6 / 8000.0},
+        "verify_attention_append": {"ms": ms_app, "note": "attention that also writes the verify tokens' K/V "
+                                                           "rows into their pages (same launch)"},
     }
     # The roofline is the single kernel with the longest launches: the attention
     # kernel (one launch per stage on this workload), ahead of each of the two

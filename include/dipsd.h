@@ -16,7 +16,9 @@
  *   dipsd_verify_attention  causal GQA attention of each user's L_i+1 verify
  *                           tokens over the user's paged bf16 KV cache;
  *   dipsd_spec_verify       speculative sampling over the vocabulary;
- *   dipsd_verify_batch      both, for one pipeline stage's users.
+ *   dipsd_verify_batch      both, for one pipeline stage's users;
+ *   *_append variants       the same, also writing the verify tokens' own
+ *                           K/V rows into their pages in the same launch.
  *
  * Conventions shared by every entry point
  *   - Pointers named d_* are device pointers, h_* host pointers.  The caller
@@ -67,6 +69,7 @@ typedef enum { DIPSD_BF16 = 0, DIPSD_F32 = 1 } dipsd_dtype;
 /* Device status bits (workspace word 0). */
 #define DIPSD_DEVERR_WAIT_TIMEOUT 1u /* a bounded mbarrier wait expired */
 #define DIPSD_DEVERR_BAD_TOKEN 2u    /* a draft token outside [0, V): treated as rejected */
+#define DIPSD_DEVERR_BAD_BLOCK 4u    /* an appended row's page id outside [0, num_blocks): row not written */
 
 /* Human-readable name of a dipsd_status value (static string). */
 const char* dipsd_status_string(int status);
@@ -171,6 +174,41 @@ int dipsd_verify_batch(int B, const int* h_members, int M,
                        const float* d_uniforms, int* d_accept_len, int* d_out_offsets,
                        int* d_out_tokens, float* d_draft_probs,
                        void* d_workspace, size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
+ * KV append inside verification (the round's state update, Sec. II-A stage 2:
+ * the verify tokens' own keys and values join each user's cache).
+ *
+ * Same as dipsd_verify_attention / dipsd_verify_batch, with the cache pages
+ * at positions C_i .. C_i+L_i (which must be allocated in the block table)
+ * not yet holding the verify tokens' rows:
+ * d_new_k, d_new_v   [sum_i (L_i+1)][Hkv][D] bf16, 16-byte aligned, users
+ *                    packed like d_q: verify token t of user i is written to
+ *                    position C_i + t (block d_block_table[i][(C_i+t)/16],
+ *                    slot (C_i+t) % 16) of d_k_cache / d_v_cache, and the
+ *                    attention of this call uses those rows (whatever the
+ *                    pages held before).  Every other cache byte is left as
+ *                    it was.
+ * Workspaces are sized by the matching *_workspace_size calls.  A page id
+ * outside [0, num_blocks) at an appended position sets
+ * DIPSD_DEVERR_BAD_BLOCK and that row is not written.
+ * ---------------------------------------------------------------------- */
+int dipsd_verify_attention_append(int B, const int* h_L, const int* h_ctx,
+                                  const void* d_q, const void* d_new_k, const void* d_new_v,
+                                  void* d_k_cache, void* d_v_cache, int num_blocks,
+                                  const int* d_block_table, int max_blocks, int Hq, int Hkv,
+                                  int D, float softmax_scale, void* d_out, void* d_workspace,
+                                  size_t workspace_bytes, void* stream);
+int dipsd_verify_batch_append(int B, const int* h_members, int M, const int* h_L_all,
+                              const int* h_ctx_all, const void* d_q, const void* d_new_k,
+                              const void* d_new_v, void* d_k_cache, void* d_v_cache,
+                              int num_blocks, const int* d_block_table_all, int max_blocks,
+                              int Hq, int Hkv, int D, float softmax_scale, void* d_attn_out,
+                              int V, int logit_dtype, const void* d_target_logits,
+                              const void* d_draft_logits, const int* d_draft_tokens,
+                              const float* d_uniforms, int* d_accept_len, int* d_out_offsets,
+                              int* d_out_tokens, float* d_draft_probs, void* d_workspace,
+                              size_t workspace_bytes, void* stream);
 
 /* ------------------------------------------------------------------------
  * Speculative verification without a caller-provided workspace.

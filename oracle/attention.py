@@ -11,8 +11,9 @@ G = Hq / Hkv (grouped-query attention, consecutive query heads share a KV
 head as in Qwen3).
 
 The KV cache is paged: page p of user i holds tokens 16p .. 16p+15 of that
-user and lives at cache block block_table[i][p].  The new tokens' K/V are
-already written into the pages when verification starts.
+user and lives at cache block block_table[i][p].  The round's state update
+writes the verify tokens' own keys and values into the pages (kv_append);
+verify_attention reads the cache as it stands after that write.
 
 Pins (tests/test_oracle_attention.py): torch's scaled_dot_product_attention
 in fp64 on the gathered, GQA-expanded tensors; kv_len = 1 gives v_0; equal
@@ -32,6 +33,31 @@ def gather_pages(cache: np.ndarray, table_row: np.ndarray, n_tokens: int) -> np.
     x = cache[blocks]                                  # [n_pages, Hkv, PAGE, D]
     x = x.transpose(1, 0, 2, 3).reshape(cache.shape[1], n_pages * PAGE, cache.shape[3])
     return x[:, :n_tokens]
+
+
+def kv_append(k_cache, v_cache, block_table, ctx, L, new_k, new_v, members=None):
+    """Writes every user's T_i new key/value rows into its pages (the verify
+    tokens join the cache in the same round, Sec. II-A stage 2).
+
+    new_k, new_v  [sum_i T_i, Hkv, D], users concatenated in batch order;
+                  verify token t of user i lands at position C_i + t, i.e.
+                  block block_table[members[i]][(C_i + t) // 16], slot
+                  (C_i + t) % 16.
+    returns       updated copies of k_cache and v_cache
+    """
+    k = np.array(k_cache, copy=True)
+    v = np.array(v_cache, copy=True)
+    members = np.arange(len(L)) if members is None else np.asarray(members)
+    n = 0
+    for i in range(len(L)):
+        row = np.asarray(block_table[int(members[i])])
+        for t in range(int(L[i]) + 1):
+            pos = int(ctx[i]) + t
+            blk, slot = int(row[pos // PAGE]), pos % PAGE
+            k[blk, :, slot, :] = new_k[n + t]
+            v[blk, :, slot, :] = new_v[n + t]
+        n += int(L[i]) + 1
+    return k, v
 
 
 def verify_attention(q, k_cache, v_cache, block_table, ctx, L, scale, members=None):

@@ -27,6 +27,12 @@
 //               lazy rescale (O in TMEM is rescaled only when a row maximum
 //               grows by more than 2^8), write P as bf16 pairs into the first
 //               32 columns of S[b] with tcgen05.st, and finally read O back.
+// KV append (p.new_k set): the T_i new rows are not read from the cache.
+// The producer patches them into every K/V tile that covers positions
+// C_i .. C_i + T_i - 1 once the tile has landed, and signals the tile on
+// k_patch / v_patch instead of k_full / v_full; the CTA with the last split
+// and the first row block of each (user, head) also writes them into the
+// pages (the round's state update).
 // KV splits: either each split writes (m, l, O) rows to global memory for
 // verify_attention_merge_kernel, or (p.cluster > 1) the splits of one row
 // block and head run as one thread-block cluster: the other ranks push their
@@ -57,7 +63,7 @@ struct TcSmem {
   static constexpr int kKOff = 0;
   static constexpr int kVOff = kKOff + kStages * kTileBytes;
   static constexpr int kBarOff = kVOff + kStages * kTileBytes;
-  static constexpr int kBytes = kBarOff + 512;
+  static constexpr int kBytes = kBarOff + 1024;  // barriers (6 kStages + 8) and the TMEM slot
   static constexpr int kAlloc = kBytes + 1024;  // slack for 1024-byte alignment
 };
 constexpr int kTcStages = TcSmem<128>::kStages;
@@ -86,7 +92,9 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
   uint64_t* pv_done = p_full + 2;      // [2]
   uint64_t* o_final = pv_done + 2;
   uint64_t* q_ready = o_final + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(q_ready + 1);
+  uint64_t* k_patch = q_ready + 1;   // [S] (each used at most once: new rows span <= 2 tiles)
+  uint64_t* v_patch = k_patch + S;   // [S]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(v_patch + S);
 
   // ---- work item
   const int item = blockIdx.x;
@@ -102,6 +110,11 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
   const int kv_begin = split * U.split_len;
   const int kv_end = min(kv_begin + U.split_len, U.kv_len);
   const int ntiles = max(0, (kv_end - kv_begin + kTcTile - 1) / kTcTile);  // 0: an empty split
+  // tile j holds new (appended) rows: keys [max(key0, C_i), min(key0 + 64, kv_len))
+  auto patched = [&](int j) {
+    const int key0 = kv_begin + j * kTcTile;
+    return p.new_k != nullptr && max(key0, U.ctx) < min(key0 + kTcTile, U.kv_len);
+  };
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -119,6 +132,10 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
     }
     mbar_init(o_final, 1);
     mbar_init(q_ready, 4);
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&k_patch[s], 1);
+      mbar_init(&v_patch[s], 1);
+    }
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
@@ -184,6 +201,57 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
       __syncwarp();
       if (lane >= kKBoxes && lane < kKBoxes + kPages) tma_load_5d(sV + voff, &tm_v, 0, 0, 0, h, bk, &v_full[st]);
       ++issued;
+      if (patched(j)) {
+        // the appended rows of this tile, straight from the input, over what
+        // the pages held (generic writes, then a proxy fence for the MMA)
+        const int key0 = kv_begin + j * kTcTile;
+        const int lo = max(key0, U.ctx), hi = min(key0 + kTcTile, U.kv_len);
+        const int n16 = (hi - lo) * (D / 8);
+        go = true;
+        if (lane == 0) go = mbar_wait(&k_full[st], (j / S) & 1, p.status);
+        if (!__shfl_sync(0xffffffffu, go, 0)) break;
+        for (int e = lane; e < n16; e += 32) {
+          const int key = lo + e / (D / 8), c = e % (D / 8), r = key - key0;
+          const uint4 v = __ldg(reinterpret_cast<const uint4*>(
+              p.new_k + (static_cast<size_t>(U.q_off + key - U.ctx) * p.Hkv + h) * D) + c);
+          *reinterpret_cast<uint4*>(sK + st * L::kTileBytes + (c >> 3) * (kTcTile * 128) + r * 128 +
+                                    (((c & 7) ^ (r & 7)) << 4)) = v;
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&k_patch[st]);
+        if (lane == 0) go = mbar_wait(&v_full[st], (j / S) & 1, p.status);
+        if (!__shfl_sync(0xffffffffu, go, 0)) break;
+        for (int e = lane; e < n16; e += 32) {
+          const int key = lo + e / (D / 8), c = e % (D / 8), r = key - key0;
+          const int r16 = r % kPage;
+          const uint4 v = __ldg(reinterpret_cast<const uint4*>(
+              p.new_v + (static_cast<size_t>(U.q_off + key - U.ctx) * p.Hkv + h) * D) + c);
+          *reinterpret_cast<uint4*>(sV + st * L::kTileBytes + (r / kPage) * L::kPageBytes + (c >> 3) * (kPage * 128) +
+                                    r16 * 128 + (((c & 7) ^ (r16 & 7)) << 4)) = v;
+        }
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&v_patch[st]);
+      }
+    }
+    // state update: the last split of the first row block writes the user's
+    // new rows of head h into the pages
+    if (p.new_k != nullptr && rb == 0 && split == U.nsplit - 1) {
+      const int n16 = U.T * (D / 8);
+      for (int e = lane; e < n16; e += 32) {
+        const int tt = e / (D / 8), c = e % (D / 8);
+        const int pos = U.ctx + tt;
+        const int blk = __ldg(bt + pos / kPage);
+        if (blk < 0 || blk >= p.num_blocks) {
+          atomicOr(p.status, kDevErrBadBlock);
+          continue;
+        }
+        const size_t dst = ((static_cast<size_t>(blk) * p.Hkv + h) * kPage + pos % kPage) * D;
+        const size_t src = (static_cast<size_t>(U.q_off + tt) * p.Hkv + h) * D;
+        reinterpret_cast<uint4*>(p.k_cache + dst)[c] = __ldg(reinterpret_cast<const uint4*>(p.new_k + src) + c);
+        reinterpret_cast<uint4*>(p.v_cache + dst)[c] = __ldg(reinterpret_cast<const uint4*>(p.new_v + src) + c);
+      }
     }
     // copies still in flight must land before the CTA can exit
     if (lane == 0)
@@ -205,7 +273,8 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
         bool did = false;
         // S[jq & 1] is free once P V of tile jq - 2 has been issued (the
         // tensor core runs one thread's MMAs in issue order)
-        if (jq < ntiles && jp >= jq - 1 && mbar_test_wait(&k_full[jq % S], (jq / S) & 1)) {
+        if (jq < ntiles && jp >= jq - 1 &&
+            (patched(jq) ? mbar_test_wait(&k_patch[jq % S], 0) : mbar_test_wait(&k_full[jq % S], (jq / S) & 1))) {
           tc_fence_after();
           const uint32_t kt = k_addr + (jq % S) * L::kTileBytes;
 #pragma unroll
@@ -219,7 +288,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
           did = true;
         }
         if (jp < jq && mbar_test_wait(&p_full[jp & 1], (jp >> 1) & 1) &&
-            mbar_test_wait(&v_full[jp % S], (jp / S) & 1)) {
+            (patched(jp) ? mbar_test_wait(&v_patch[jp % S], 0) : mbar_test_wait(&v_full[jp % S], (jp / S) & 1))) {
           tc_fence_after();
           const uint32_t vt = v_addr + (jp % S) * L::kTileBytes;
           const uint32_t pt = tS0 + (jp & 1) * kTcTile;  // P: 32 columns of bf16 pairs

@@ -286,6 +286,12 @@ void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int
   pl.ws_bytes = part ? align_up(part * sizeof(float2), 256) + align_up(part * D * sizeof(float), 256) : 0;
 }
 
+// KV-append inputs of one call (all null: the cache already holds the rows).
+struct KvAppend {
+  const void* new_k = nullptr;
+  const void* new_v = nullptr;
+};
+
 template <int CAP>
 void fill_attn_params(AttnParams<CAP>& p, const AttnPlan& pl, const void* q, void* out, const int* bt,
                       int max_blocks, float scale, unsigned* status, uint8_t* region) {
@@ -328,9 +334,14 @@ int launch_attention_tc_t(const AttnPlan& pl, const AttnParams<CAP>& p, const CU
 template <int CAP>
 int run_attention_cap(const AttnPlan& pl, const void* q, const void* kc, const void* vc, int num_blocks,
                       const int* bt, int max_blocks, float scale, void* out, unsigned* status,
-                      uint8_t* region, cudaStream_t s, bool pdl) {
+                      uint8_t* region, cudaStream_t s, bool pdl, const KvAppend& app) {
   static thread_local AttnParams<CAP> p;
   fill_attn_params<CAP>(p, pl, q, out, bt, max_blocks, scale, status, region);
+  p.new_k = static_cast<const __nv_bfloat16*>(app.new_k);
+  p.new_v = static_cast<const __nv_bfloat16*>(app.new_v);
+  p.k_cache = static_cast<__nv_bfloat16*>(const_cast<void*>(kc));
+  p.v_cache = static_cast<__nv_bfloat16*>(const_cast<void*>(vc));
+  p.num_blocks = num_blocks;
   alignas(64) CUtensorMap tk, tv;
   if (!encode_cache_map(&tk, kc, num_blocks, pl.Hkv, pl.D, false) ||
       !encode_cache_map(&tv, vc, num_blocks, pl.Hkv, pl.D, true))
@@ -341,12 +352,19 @@ int run_attention_cap(const AttnPlan& pl, const void* q, const void* kc, const v
 
 int run_attention(const AttnPlan& pl, const void* q, const void* kc, const void* vc, int num_blocks,
                   const int* bt, int max_blocks, float scale, void* out, unsigned* status, uint8_t* region,
-                  cudaStream_t s, bool pdl) {
+                  cudaStream_t s, bool pdl, const KvAppend& app = KvAppend{}) {
   if (pl.B <= kCapSmall)
     return run_attention_cap<kCapSmall>(pl, q, kc, vc, num_blocks, bt, max_blocks, scale, out, status,
-                                        region, s, pdl);
+                                        region, s, pdl, app);
   return run_attention_cap<kCapLarge>(pl, q, kc, vc, num_blocks, bt, max_blocks, scale, out, status,
-                                      region, s, pdl);
+                                      region, s, pdl, app);
+}
+
+int check_append(const void* new_k, const void* new_v, const void* q) {
+  if (!new_k || !new_v) return DIPSD_ERR_INVALID_ARG;
+  if (!aligned(new_k, 16) || !aligned(new_v, 16)) return DIPSD_ERR_INVALID_ARG;
+  if (new_k == new_v || new_k == q || new_v == q) return DIPSD_ERR_INVALID_ARG;
+  return DIPSD_OK;
 }
 
 int check_attn_buffers(const void* q, const void* kc, const void* vc, int num_blocks, const int* bt,
@@ -613,10 +631,10 @@ size_t dipsd_verify_attention_workspace_size(int B, const int* h_L, const int* h
   return kHeaderBytes + pl.ws_bytes;
 }
 
-int dipsd_verify_attention(int B, const int* h_L, const int* h_ctx, const void* d_q, const void* d_k_cache,
-                           const void* d_v_cache, int num_blocks, const int* d_block_table, int max_blocks,
-                           int Hq, int Hkv, int D, float softmax_scale, void* d_out, void* d_workspace,
-                           size_t workspace_bytes, void* stream) {
+static int verify_attention_impl(int B, const int* h_L, const int* h_ctx, const void* d_q, const void* d_k_cache,
+                                 const void* d_v_cache, int num_blocks, const int* d_block_table, int max_blocks,
+                                 int Hq, int Hkv, int D, float softmax_scale, void* d_out, void* d_workspace,
+                                 size_t workspace_bytes, void* stream, const KvAppend& app) {
   int st = check_attn_users(B, h_L, h_ctx, Hq, Hkv, D);
   if (st != DIPSD_OK) return st;
   st = check_attn_buffers(d_q, d_k_cache, d_v_cache, num_blocks, d_block_table, max_blocks, d_out, B, h_L,
@@ -630,8 +648,31 @@ int dipsd_verify_attention(int B, const int* h_L, const int* h_ctx, const void* 
   if (st != DIPSD_OK) return st;
   uint8_t* ws = static_cast<uint8_t*>(d_workspace);
   st = run_attention(pl, d_q, d_k_cache, d_v_cache, num_blocks, d_block_table, max_blocks, softmax_scale, d_out,
-                     reinterpret_cast<unsigned*>(ws), ws + kHeaderBytes, static_cast<cudaStream_t>(stream), true);
+                     reinterpret_cast<unsigned*>(ws), ws + kHeaderBytes, static_cast<cudaStream_t>(stream), true,
+                     app);
   return st != DIPSD_OK ? st : cuda_status();
+}
+
+int dipsd_verify_attention(int B, const int* h_L, const int* h_ctx, const void* d_q, const void* d_k_cache,
+                           const void* d_v_cache, int num_blocks, const int* d_block_table, int max_blocks,
+                           int Hq, int Hkv, int D, float softmax_scale, void* d_out, void* d_workspace,
+                           size_t workspace_bytes, void* stream) {
+  return verify_attention_impl(B, h_L, h_ctx, d_q, d_k_cache, d_v_cache, num_blocks, d_block_table, max_blocks, Hq,
+                               Hkv, D, softmax_scale, d_out, d_workspace, workspace_bytes, stream, KvAppend{});
+}
+
+int dipsd_verify_attention_append(int B, const int* h_L, const int* h_ctx, const void* d_q, const void* d_new_k,
+                                  const void* d_new_v, void* d_k_cache, void* d_v_cache, int num_blocks,
+                                  const int* d_block_table, int max_blocks, int Hq, int Hkv, int D,
+                                  float softmax_scale, void* d_out, void* d_workspace, size_t workspace_bytes,
+                                  void* stream) {
+  const int st = check_append(d_new_k, d_new_v, d_q);
+  if (st != DIPSD_OK) return st;
+  KvAppend app;
+  app.new_k = d_new_k;
+  app.new_v = d_new_v;
+  return verify_attention_impl(B, h_L, h_ctx, d_q, d_k_cache, d_v_cache, num_blocks, d_block_table, max_blocks, Hq,
+                               Hkv, D, softmax_scale, d_out, d_workspace, workspace_bytes, stream, app);
 }
 
 size_t dipsd_spec_verify_workspace_size(int B, const int* h_L, int V) {
@@ -724,13 +765,14 @@ size_t dipsd_verify_batch_workspace_size(int B, const int* h_members, int M, con
   return kHeaderBytes + align_up(ap.ws_bytes, 256) + spec_ws_need(B, L.data(), V);
 }
 
-int dipsd_verify_batch(int B, const int* h_members, int M, const int* h_L_all, const int* h_ctx_all,
-                       const void* d_q, const void* d_k_cache, const void* d_v_cache, int num_blocks,
-                       const int* d_block_table_all, int max_blocks, int Hq, int Hkv, int D, float softmax_scale,
-                       void* d_attn_out, int V, int logit_dtype, const void* d_target_logits,
-                       const void* d_draft_logits, const int* d_draft_tokens, const float* d_uniforms,
-                       int* d_accept_len, int* d_out_offsets, int* d_out_tokens, float* d_draft_probs,
-                       void* d_workspace, size_t workspace_bytes, void* stream) {
+static int verify_batch_impl(int B, const int* h_members, int M, const int* h_L_all, const int* h_ctx_all,
+                             const void* d_q, const void* d_k_cache, const void* d_v_cache, int num_blocks,
+                             const int* d_block_table_all, int max_blocks, int Hq, int Hkv, int D,
+                             float softmax_scale, void* d_attn_out, int V, int logit_dtype,
+                             const void* d_target_logits, const void* d_draft_logits, const int* d_draft_tokens,
+                             const float* d_uniforms, int* d_accept_len, int* d_out_offsets, int* d_out_tokens,
+                             float* d_draft_probs, void* d_workspace, size_t workspace_bytes, void* stream,
+                             const KvAppend& app) {
   std::vector<int> L, ctx;
   int st = gather_members(B, h_members, M, h_L_all, h_ctx_all, L, ctx);
   if (st != DIPSD_OK) return st;
@@ -760,11 +802,42 @@ int dipsd_verify_batch(int B, const int* h_members, int M, const int* h_L_all, c
   unsigned* status = reinterpret_cast<unsigned*>(ws);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   st = run_attention(ap, d_q, d_k_cache, d_v_cache, num_blocks, d_block_table_all, max_blocks, softmax_scale,
-                     d_attn_out, status, ws + kHeaderBytes, s, true);
+                     d_attn_out, status, ws + kHeaderBytes, s, true, app);
   if (st != DIPSD_OK) return st;
   st = run_spec(sp, logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
                 d_out_offsets, d_out_tokens, d_draft_probs, status, ws + kHeaderBytes + attn_region, s, true);
   return st != DIPSD_OK ? st : cuda_status();
+}
+
+int dipsd_verify_batch(int B, const int* h_members, int M, const int* h_L_all, const int* h_ctx_all,
+                       const void* d_q, const void* d_k_cache, const void* d_v_cache, int num_blocks,
+                       const int* d_block_table_all, int max_blocks, int Hq, int Hkv, int D, float softmax_scale,
+                       void* d_attn_out, int V, int logit_dtype, const void* d_target_logits,
+                       const void* d_draft_logits, const int* d_draft_tokens, const float* d_uniforms,
+                       int* d_accept_len, int* d_out_offsets, int* d_out_tokens, float* d_draft_probs,
+                       void* d_workspace, size_t workspace_bytes, void* stream) {
+  return verify_batch_impl(B, h_members, M, h_L_all, h_ctx_all, d_q, d_k_cache, d_v_cache, num_blocks,
+                           d_block_table_all, max_blocks, Hq, Hkv, D, softmax_scale, d_attn_out, V, logit_dtype,
+                           d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len, d_out_offsets,
+                           d_out_tokens, d_draft_probs, d_workspace, workspace_bytes, stream, KvAppend{});
+}
+
+int dipsd_verify_batch_append(int B, const int* h_members, int M, const int* h_L_all, const int* h_ctx_all,
+                              const void* d_q, const void* d_new_k, const void* d_new_v, void* d_k_cache,
+                              void* d_v_cache, int num_blocks, const int* d_block_table_all, int max_blocks, int Hq,
+                              int Hkv, int D, float softmax_scale, void* d_attn_out, int V, int logit_dtype,
+                              const void* d_target_logits, const void* d_draft_logits, const int* d_draft_tokens,
+                              const float* d_uniforms, int* d_accept_len, int* d_out_offsets, int* d_out_tokens,
+                              float* d_draft_probs, void* d_workspace, size_t workspace_bytes, void* stream) {
+  const int st = check_append(d_new_k, d_new_v, d_q);
+  if (st != DIPSD_OK) return st;
+  KvAppend app;
+  app.new_k = d_new_k;
+  app.new_v = d_new_v;
+  return verify_batch_impl(B, h_members, M, h_L_all, h_ctx_all, d_q, d_k_cache, d_v_cache, num_blocks,
+                           d_block_table_all, max_blocks, Hq, Hkv, D, softmax_scale, d_attn_out, V, logit_dtype,
+                           d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len, d_out_offsets,
+                           d_out_tokens, d_draft_probs, d_workspace, workspace_bytes, stream, app);
 }
 
 }  // extern "C"

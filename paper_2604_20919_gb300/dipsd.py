@@ -26,12 +26,14 @@ MAX_USERS = 512
 MAX_DRAFT = 31
 DEVERR_WAIT_TIMEOUT = 1
 DEVERR_BAD_TOKEN = 2
+DEVERR_BAD_BLOCK = 4
 
 EXPORTS = (
     "dipsd_status_string", "dipsd_abi_version", "dipsd_launch_count",
     "dipsd_verify_attention_workspace_size", "dipsd_verify_attention",
     "dipsd_spec_verify_workspace_size", "dipsd_spec_verify",
     "dipsd_verify_batch_workspace_size", "dipsd_verify_batch", "dipsd_spec_verify_noalloc",
+    "dipsd_verify_attention_append", "dipsd_verify_batch_append",
 )
 NOALLOC_MAX_POSITIONS = 4096
 
@@ -75,6 +77,13 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.dipsd_verify_batch.argtypes = [_i, _i32p, _i, _i32p, _i32p, _vp, _vp, _vp, _i, _vp, _i, _i, _i, _i,
                                        ctypes.c_float, _vp, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
                                        _vp, _sz, _vp]
+    lib.dipsd_verify_attention_append.restype = _i
+    lib.dipsd_verify_attention_append.argtypes = [_i, _i32p, _i32p, _vp, _vp, _vp, _vp, _vp, _i, _vp, _i, _i, _i,
+                                                  _i, ctypes.c_float, _vp, _vp, _sz, _vp]
+    lib.dipsd_verify_batch_append.restype = _i
+    lib.dipsd_verify_batch_append.argtypes = [_i, _i32p, _i, _i32p, _i32p, _vp, _vp, _vp, _vp, _vp, _i, _vp, _i,
+                                              _i, _i, _i, ctypes.c_float, _vp, _i, _i, _vp, _vp, _vp, _vp, _vp,
+                                              _vp, _vp, _vp, _vp, _sz, _vp]
     lib.dipsd_spec_verify_noalloc.restype = _i
     lib.dipsd_spec_verify_noalloc.argtypes = [_i, _i32p, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]
     _lib = lib
@@ -170,6 +179,37 @@ def dipsd_verify_attention(L, ctx, q, k_cache, v_cache, block_table, softmax_sca
     return out
 
 
+def dipsd_verify_attention_append(L, ctx, q, new_k, new_v, k_cache, v_cache, block_table, softmax_scale: float,
+                                  out=None, ws=None, stream=None) -> torch.Tensor:
+    """As dipsd_verify_attention, first writing the verify tokens' K/V rows
+    (new_k, new_v [sum T][Hkv][D]) into their pages (positions C_i + t)."""
+    lib = load()
+    a, pa = _host_i32(L)
+    b, pb = _host_i32(ctx)
+    sum_t = int((a + 1).sum())
+    nb, Hkv, page, D = k_cache.shape
+    Hq = q.shape[1]
+    if page != PAGE_SIZE or tuple(q.shape) != (sum_t, Hq, D) or tuple(v_cache.shape) != tuple(k_cache.shape):
+        raise ValueError("shape mismatch between q, caches and lengths")
+    if tuple(new_k.shape) != (sum_t, Hkv, D) or tuple(new_v.shape) != (sum_t, Hkv, D):
+        raise ValueError("new_k / new_v must be [sum T][Hkv][D]")
+    if block_table.dim() != 2 or block_table.shape[0] != len(a):
+        raise ValueError("block_table must be [B][max_blocks]")
+    if out is None:
+        out = torch.empty_like(q)
+    if ws is None:
+        ws = workspace(dipsd_verify_attention_workspace_size(a, b, Hq, Hkv, D), q.device)
+    st = lib.dipsd_verify_attention_append(len(a), pa, pb, _dptr(q, "q", torch.bfloat16),
+                                           _dptr(new_k, "new_k", torch.bfloat16), _dptr(new_v, "new_v", torch.bfloat16),
+                                           _dptr(k_cache, "k_cache", torch.bfloat16),
+                                           _dptr(v_cache, "v_cache", torch.bfloat16), nb,
+                                           _dptr(block_table, "block_table", torch.int32), block_table.shape[1],
+                                           Hq, Hkv, D, float(softmax_scale), _dptr(out, "out", torch.bfloat16),
+                                           _dptr(ws, "workspace"), ws.numel(), _stream(stream))
+    _check(st, "dipsd_verify_attention_append")
+    return out
+
+
 # ---------------------------------------------------------- spec verification
 def dipsd_spec_verify_workspace_size(L, V: int) -> int:
     a, pa = _host_i32(L)
@@ -221,9 +261,8 @@ def dipsd_verify_batch_workspace_size(members, L_all, ctx_all, Hq, Hkv, D, V) ->
     return int(load().dipsd_verify_batch_workspace_size(len(m), pm, len(a), pa, pb, Hq, Hkv, D, V))
 
 
-def dipsd_verify_batch(members, L_all, ctx_all, q, k_cache, v_cache, block_table_all, softmax_scale,
-                       target_logits, draft_logits, draft_tokens, uniforms, attn_out=None, outputs=None,
-                       ws=None, stream=None):
+def _verify_batch(members, L_all, ctx_all, q, k_cache, v_cache, block_table_all, softmax_scale, target_logits,
+                  draft_logits, draft_tokens, uniforms, attn_out, outputs, ws, stream, new_kv):
     """Attention then speculative verification for the users `members` of one stage.
 
     Returns (attn_out, accept_len, out_offsets, out_tokens, draft_probs).
@@ -245,7 +284,17 @@ def dipsd_verify_batch(members, L_all, ctx_all, q, k_cache, v_cache, block_table
     acc, offs, toks, probs = outputs if outputs is not None else spec_outputs(Lb, q.device)
     if ws is None:
         ws = workspace(dipsd_verify_batch_workspace_size(m, a, b, Hq, Hkv, D, V), q.device)
-    st = lib.dipsd_verify_batch(len(m), pm, len(a), pa, pb, _dptr(q, "q", torch.bfloat16),
+    if new_kv is not None:
+        new_k, new_v = new_kv
+        if tuple(new_k.shape) != (sum_t, Hkv, D) or tuple(new_v.shape) != (sum_t, Hkv, D):
+            raise ValueError("new_k / new_v must be [sum T][Hkv][D]")
+        fn, name = lib.dipsd_verify_batch_append, "dipsd_verify_batch_append"
+        head = (_dptr(q, "q", torch.bfloat16), _dptr(new_k, "new_k", torch.bfloat16),
+                _dptr(new_v, "new_v", torch.bfloat16))
+    else:
+        fn, name = lib.dipsd_verify_batch, "dipsd_verify_batch"
+        head = (_dptr(q, "q", torch.bfloat16),)
+    st = fn(len(m), pm, len(a), pa, pb, *head,
                                 _dptr(k_cache, "k_cache", torch.bfloat16), _dptr(v_cache, "v_cache", torch.bfloat16),
                                 nb, _dptr(block_table_all, "block_table", torch.int32), block_table_all.shape[1],
                                 Hq, Hkv, D, float(softmax_scale), _dptr(attn_out, "attn_out", torch.bfloat16), V,
@@ -256,5 +305,25 @@ def dipsd_verify_batch(members, L_all, ctx_all, q, k_cache, v_cache, block_table
                                 _dptr(acc, "accept_len", torch.int32), _dptr(offs, "out_offsets", torch.int32),
                                 _dptr(toks, "out_tokens", torch.int32), _dptr(probs, "draft_probs", torch.float32),
                                 _dptr(ws, "workspace"), ws.numel(), _stream(stream))
-    _check(st, "dipsd_verify_batch")
+    _check(st, name)
     return attn_out, acc, offs, toks, probs
+
+
+def dipsd_verify_batch(members, L_all, ctx_all, q, k_cache, v_cache, block_table_all, softmax_scale,
+                       target_logits, draft_logits, draft_tokens, uniforms, attn_out=None, outputs=None,
+                       ws=None, stream=None):
+    """Attention then speculative verification for the users `members` of one stage.
+
+    Returns (attn_out, accept_len, out_offsets, out_tokens, draft_probs).
+    """
+    return _verify_batch(members, L_all, ctx_all, q, k_cache, v_cache, block_table_all, softmax_scale,
+                         target_logits, draft_logits, draft_tokens, uniforms, attn_out, outputs, ws, stream, None)
+
+
+def dipsd_verify_batch_append(members, L_all, ctx_all, q, new_k, new_v, k_cache, v_cache, block_table_all,
+                              softmax_scale, target_logits, draft_logits, draft_tokens, uniforms, attn_out=None,
+                              outputs=None, ws=None, stream=None):
+    """As dipsd_verify_batch, first writing the verify tokens' K/V rows into their pages."""
+    return _verify_batch(members, L_all, ctx_all, q, k_cache, v_cache, block_table_all, softmax_scale,
+                         target_logits, draft_logits, draft_tokens, uniforms, attn_out, outputs, ws, stream,
+                         (new_k, new_v))

@@ -117,3 +117,63 @@ def test_members_select_block_table_rows():
     q_sub = np.concatenate([q[5:6], q[0:2]])
     sub = verify_attention(q_sub, kc, vc, bt, [33, 20], [0, 1], 0.4, members=[2, 0])
     np.testing.assert_array_equal(sub, np.concatenate([full[5:6], full[0:2]]))
+
+
+def _new_rows(Ks, ctx, L):
+    """[sum T, Hkv, D]: each user's verify-token rows, read from the logical K/V."""
+    return np.concatenate([Ks[i][:, ctx[i]:ctx[i] + L[i] + 1].transpose(1, 0, 2) for i in range(len(L))])
+
+
+def test_kv_append_restores_poisoned_slots_exactly():
+    """Poison the verify tokens' slots, append their rows: the cache the test
+    scattered itself comes back bit for bit, and attention on it still matches
+    torch's SDPA."""
+    from oracle import kv_append
+    rng = np.random.default_rng(31)
+    L, ctx = [3, 0, 5], [17, 0, 40]
+    q, kc, vc, bt, Ks, Vs = _paged_problem(rng, L, ctx, 8, 2, 16)
+    pk, pv = kc.copy(), vc.copy()
+    for i in range(len(L)):
+        for t in range(L[i] + 1):
+            pos = ctx[i] + t
+            pk[bt[i, pos // PAGE], :, pos % PAGE] = np.nan
+            pv[bt[i, pos // PAGE], :, pos % PAGE] = np.nan
+    k2, v2 = kv_append(pk, pv, bt, ctx, L, _new_rows(Ks, ctx, L), _new_rows(Vs, ctx, L))
+    assert np.array_equal(k2, kc) and np.array_equal(v2, vc)
+    o = verify_attention(q, k2, v2, bt, ctx, L, 0.25)
+    np.testing.assert_allclose(o, _sdpa_reference(q, Ks, Vs, ctx, L, 0.25, 4), rtol=0, atol=1e-12)
+
+
+def test_kv_append_touches_only_the_verify_slots():
+    from oracle import kv_append
+    rng = np.random.default_rng(32)
+    L, ctx = [2, 4], [30, 3]
+    _, kc, vc, bt, Ks, Vs = _paged_problem(rng, L, ctx, 4, 1, 8)
+    nk = rng.normal(size=(sum(l + 1 for l in L), 1, 8))
+    nv = rng.normal(size=nk.shape)
+    k2, v2 = kv_append(kc, vc, bt, ctx, L, nk, nv)
+    touched = np.zeros(kc.shape[:1] + kc.shape[2:3], dtype=bool)  # [block, slot]
+    n = 0
+    for i in range(len(L)):
+        for t in range(L[i] + 1):
+            pos = ctx[i] + t
+            blk, slot = bt[i, pos // PAGE], pos % PAGE
+            touched[blk, slot] = True
+            assert np.array_equal(k2[blk, :, slot], nk[n]) and np.array_equal(v2[blk, :, slot], nv[n])
+            n += 1
+    untouched = ~touched
+    assert np.array_equal(k2.transpose(0, 2, 1, 3)[untouched], kc.transpose(0, 2, 1, 3)[untouched])
+    assert np.array_equal(v2.transpose(0, 2, 1, 3)[untouched], vc.transpose(0, 2, 1, 3)[untouched])
+
+
+def test_kv_append_follows_members():
+    """With members, user i writes through block-table row members[i]."""
+    from oracle import kv_append
+    rng = np.random.default_rng(33)
+    L, ctx = [1, 2], [5, 20]
+    _, kc, vc, bt, Ks, Vs = _paged_problem(rng, L, ctx, 2, 1, 8)
+    bt_perm = bt[::-1].copy()  # table rows in the other order
+    nk, nv = _new_rows(Ks, ctx, L), _new_rows(Vs, ctx, L)
+    a = kv_append(kc, vc, bt, ctx, L, nk, nv)
+    b = kv_append(kc, vc, bt_perm, ctx, L, nk, nv, members=[1, 0])
+    assert np.array_equal(a[0], b[0]) and np.array_equal(a[1], b[1])
