@@ -123,6 +123,13 @@ def spec_bytes(b):
     return (b.sum_T + b.sum_L) * b.V * el
 
 
+def sparse_bytes(b, K=64):
+    """Algorithmic bytes of one sparse-payload launch: one pass over every
+    target-logit row, plus the table (K entries of 8 bytes) and log q(d) per draft row."""
+    el = 2 if b.logit_dtype == "bf16" else 4
+    return b.sum_T * b.V * el + b.sum_L * (8 * K + 4)
+
+
 def source_hash(paths):
     h = hashlib.sha256()
     for p in paths:
@@ -269,6 +276,18 @@ def run_dipsd(args):
     new_k = b.k_cache[blk, :, slot].contiguous()
     new_v = b.v_cache[blk, :, slot].contiguous()
 
+    # sparse draft payload of the same batch (K = 64 table entries per draft row)
+    from workloads import make_sparse_draft
+    sdraft = make_sparse_draft(b, 64, seed=args.seed)
+    sd_dev = {k: getattr(sdraft, k).to(dev) for k in ("draft_tokens", "draft_logq", "topk_idx", "topk_q")}
+    sp_outs = dipsd.spec_outputs(b.L, dev)
+    ws_sp = dipsd.workspace(dipsd.dipsd_spec_verify_sparse_workspace_size(b.L, b.V), dev)
+
+    def spec_sparse(k):
+        c = copies[k % R]
+        dipsd.dipsd_spec_verify_sparse(b.L, c["z"], sd_dev["draft_tokens"], sd_dev["draft_logq"], sd_dev["topk_idx"],
+                                       sd_dev["topk_q"], c["u"], outputs=sp_outs, ws=ws_sp)
+
     def attn_append(k):
         c = copies[k % R]
         dipsd.dipsd_verify_attention_append(b.L, b.ctx, c["q"], new_k, new_v, c["kc"], c["vc"], bt, b.scale,
@@ -331,6 +350,7 @@ def run_dipsd(args):
     g_attn, _ = graph_of(attn_only, n_steps)
     g_spec, _ = graph_of(spec_only, n_steps)
     g_app, _ = graph_of(attn_append, n_steps)
+    g_sps, _ = graph_of(spec_sparse, n_steps)
 
     sampler = ClockSampler(local)
     sampler.start()
@@ -338,6 +358,7 @@ def run_dipsd(args):
     ms_attn = timed(g_attn, n_steps)
     ms_spec = timed(g_spec, n_steps)
     ms_app = timed(g_app, n_steps)
+    ms_sps = timed(g_sps, n_steps)
     lat_step = cold_latency(step, min(args.steps, 50))
 
     # end to end through the same call: every step copies its inputs from pinned
@@ -416,6 +437,10 @@ def run_dipsd(args):
                         "frac_of_8000": s_bytes / ms_spec / 1e6 / 8000.0},
         "verify_attention_append": {"ms": ms_app, "note": "attention that also writes the verify tokens' K/V "
                                                            "rows into their pages (same launch)"},
+        "spec_verify_sparse": {"ms": ms_sps, "alg_bytes": sparse_bytes(b),
+                               "gbs": sparse_bytes(b) / ms_sps / 1e6,
+                               "frac_of_measured_hbm": sparse_bytes(b) / ms_sps / 1e6 / hbm_peak,
+                               "note": "sparse draft payload, K = 64 table entries per draft row"},
     }
     # The roofline is the single kernel with the longest launches: the attention
     # kernel (one launch per stage on this workload), ahead of each of the two

@@ -18,7 +18,10 @@
  *   dipsd_spec_verify       speculative sampling over the vocabulary;
  *   dipsd_verify_batch      both, for one pipeline stage's users;
  *   *_append variants       the same, also writing the verify tokens' own
- *                           K/V rows into their pages in the same launch.
+ *                           K/V rows into their pages in the same launch;
+ *   dipsd_spec_verify_sparse  speculative sampling from a sparse draft
+ *                           payload (draft-token log-probabilities and a
+ *                           top-K draft distribution).
  *
  * Conventions shared by every entry point
  *   - Pointers named d_* are device pointers, h_* host pointers.  The caller
@@ -150,6 +153,34 @@ int dipsd_spec_verify(int B, const int* h_L, int V, int logit_dtype,
                       int* d_accept_len, int* d_out_offsets, int* d_out_tokens,
                       float* d_draft_probs, void* d_workspace, size_t workspace_bytes,
                       void* stream);
+
+/* ------------------------------------------------------------------------
+ * Speculative verification from a sparse draft payload (Sec. II-A: the device
+ * sends the drafted tokens and, when the protocol needs it, a small amount of
+ * probability information such as the draft tokens' log-probabilities).
+ *
+ * As dipsd_spec_verify without draft logits.  For draft position t of user i
+ * (draft row r = sum_{j<i} L_j + t) the draft distribution q_r is the table
+ * (d_topk_idx[r][k], d_topk_q[r][k]), k < K: q_r(idx) = q, 0 for every token
+ * not in the table (exact for a device that samples from its own top K).
+ *   accepted iff u_acc(t) * exp(d_draft_logq[r]) < p_t(d);
+ *   residual max(0, p_a - q_a) over the whole vocabulary.
+ * K                 1..64;  d_topk_idx [sum L][K] int32 (distinct tokens;
+ *                   entries outside [0, V) are ignored and set
+ *                   DIPSD_DEVERR_BAD_TOKEN), d_topk_q [sum L][K] fp32 >= 0,
+ *                   d_draft_logq [sum L] fp32.
+ * Only the target logit rows are read.  Rows must be 16-byte aligned
+ * (V * elem % 16 == 0), else DIPSD_ERR_UNSUPPORTED.  d_draft_probs gets
+ * (p_t(d), exp(draft_logq)).
+ * ---------------------------------------------------------------------- */
+size_t dipsd_spec_verify_sparse_workspace_size(int B, const int* h_L, int V);
+int dipsd_spec_verify_sparse(int B, const int* h_L, int V, int K, int logit_dtype,
+                             const void* d_target_logits, const int* d_draft_tokens,
+                             const float* d_draft_logq, const int* d_topk_idx,
+                             const float* d_topk_q, const float* d_uniforms,
+                             int* d_accept_len, int* d_out_offsets, int* d_out_tokens,
+                             float* d_draft_probs, void* d_workspace, size_t workspace_bytes,
+                             void* stream);
 
 /* ------------------------------------------------------------------------
  * One pipeline stage: the users of batch n (Sec. III-C, B_n(x)) verified

@@ -10,6 +10,8 @@ computes in one batch-verification round (paper Sec. II-A, stage 2):
   * spec_verify.spec_verify    -- speculative sampling: accept/reject each
     draft token, truncate at the first rejection, resample from the residual
     or from p at the bonus position, pack the emitted tokens.
+  * spec_verify.spec_verify_sparse -- the same from a sparse draft payload
+    (draft-token log-probabilities and a top-K draft distribution).
 
 Only tests/, __graft_entry__.smoke() and bench.py's cpu_baseline / reference
 leg may import this package.  It shares no code with the CUDA library and
@@ -18,6 +20,6 @@ closed forms, invariants, library routines or brute force (see each
 function's docstring for its pin).
 """
 from .attention import kv_append, verify_attention
-from .spec_verify import softmax, inverse_cdf, spec_verify, decision_margins
+from .spec_verify import softmax, inverse_cdf, spec_verify, spec_verify_sparse, decision_margins
 
-__all__ = ["kv_append", "verify_attention", "softmax", "inverse_cdf", "spec_verify", "decision_margins"]
+__all__ = ["kv_append", "verify_attention", "softmax", "inverse_cdf", "spec_verify", "spec_verify_sparse", "decision_margins"]

@@ -27,6 +27,9 @@ Readings where the method leaves a choice (each listed in the design doc):
     cumsum(w)[k] > u * sum(w); if rounding leaves none, the last k with w_k > 0;
   * a residual with no positive mass falls back to p_a.
 
+spec_verify_sparse takes the draft distribution as a sparse table and the
+draft tokens' probabilities as given numbers; its steps are the same.
+
 Pins (tests/test_oracle_spec.py): scipy softmax; exact brute force of the
 whole output law on tiny vocabularies against the closed form
 prod_t min(p_t, q_t) * (residual or p); Monte Carlo chi-square of the
@@ -85,12 +88,42 @@ def spec_verify(L, target_logits, draft_logits, draft_tokens, uniforms):
       margin_resample [B]      distance of u_res from the chosen token's CDF cell edges
       resample_mass [B]        total mass of the distribution sampled at a_i
     """
-    L = np.asarray(L, dtype=np.int64)
-    B = L.shape[0]
-    uni = np.asarray(uniforms, dtype=np.float64)
     dt = np.asarray(draft_tokens, dtype=np.int64)
     p = softmax(target_logits)
     q = softmax(draft_logits) if len(dt) else np.zeros((0, p.shape[1]))
+    q_d = q[np.arange(len(dt)), dt] if len(dt) else np.zeros(0)
+    return _verify(L, p, q, q_d, dt, uniforms)
+
+
+def spec_verify_sparse(L, target_logits, draft_tokens, draft_logq, topk_idx, topk_q, uniforms):
+    """Speculative verification from a sparse draft payload (Sec. II-A: the
+    device sends the drafted tokens and a small amount of probability
+    information, e.g. draft-token log-probabilities).
+
+    The draft distribution of draft position r is the table (topk_idx[r],
+    topk_q[r]): q_r(topk_idx[r, j]) = topk_q[r, j] and 0 elsewhere (exact for
+    a device that samples from its top K).  The acceptance test reads
+    q_r(d) = exp(draft_logq[r]); the residual is max(0, p - q_r) over the whole
+    vocabulary.  Everything else is spec_verify.
+
+    draft_logq [sum_i L_i]; topk_idx, topk_q [sum_i L_i, K] (distinct indices)
+    """
+    dt = np.asarray(draft_tokens, dtype=np.int64)
+    p = softmax(target_logits)
+    idx = np.asarray(topk_idx, dtype=np.int64)
+    q = np.zeros((len(dt), p.shape[1]))
+    for r in range(len(dt)):
+        q[r, idx[r]] = np.asarray(topk_q[r], dtype=np.float64)
+    q_d = np.exp(np.asarray(draft_logq, dtype=np.float64))
+    return _verify(L, p, q, q_d, dt, uniforms)
+
+
+def _verify(L, p, q, q_d_all, dt, uniforms):
+    """Steps 2-5 for target distributions p [sum T, V], draft distributions
+    q [sum L, V] and the draft tokens' draft probabilities q_d_all [sum L]."""
+    L = np.asarray(L, dtype=np.int64)
+    B = L.shape[0]
+    uni = np.asarray(uniforms, dtype=np.float64)
     sT = p.shape[0]
 
     accepted = np.zeros(sT, dtype=bool)
@@ -108,7 +141,7 @@ def spec_verify(L, target_logits, draft_logits, draft_tokens, uniforms):
         # step 2: acceptance test at every draft position
         for t in range(Li):
             d = dt[lo + t]
-            pd, qd = p[qo + t, d], q[lo + t, d]
+            pd, qd = p[qo + t, d], q_d_all[lo + t]
             p_d[qo + t], q_d[qo + t] = pd, qd
             accepted[qo + t] = uni[qo + t, 0] * qd < pd
             margin_accept[qo + t] = abs(uni[qo + t, 0] - pd / qd) if qd > 0 else np.inf

@@ -386,6 +386,7 @@ struct SpecPlan {
   int nk1 = 0, nk2 = 0;  // register path: vectors per lane and segment (0 = generic path)
   int nseg1 = 0, nseg2 = 0, n_items1 = 0, n_items2 = 0;
   int sum_t = 0, sum_l = 0;
+  bool sparse = false;  // sparse draft payload: no draft logit rows
   std::vector<int> q_off, l_off;
   size_t off_flags = 0, off_part1 = 0, off_part2 = 0;
   size_t ws_bytes = 0;  // spec region only
@@ -425,8 +426,9 @@ int pick_nk(const int (&opts)[K], long long rows, int nvec, int sms) {
   return opts[K - 1];
 }
 
-void plan_spec(int B, const int* L, int V, int elem, bool vec_ok, int sms, SpecPlan& pl) {
+void plan_spec(int B, const int* L, int V, int elem, bool vec_ok, int sms, SpecPlan& pl, bool sparse = false) {
   pl.B = B; pl.V = V;
+  pl.sparse = sparse;
   pl.vec = vec_ok ? 16 / elem : 1;
   pl.nvec = V / pl.vec;
   pl.cl1 = cluster_for(pl.nvec);
@@ -446,10 +448,17 @@ void plan_spec(int B, const int* L, int V, int elem, bool vec_ok, int sms, SpecP
   o += align_up(pl.sum_t, 256);
   pl.off_part1 = pl.off_part2 = o;
   if (vec_ok) {
-    const int nk1 = pick_nk(kNk1, pl.sum_t + pl.sum_l, pl.nvec, sms);
-    const int nk2 = pick_nk(kNk2, B, pl.nvec, sms);
+    const int rows = pl.sum_t + (sparse ? 0 : pl.sum_l);
+    int nk1 = pick_nk(kNk1, rows, pl.nvec, sms);
+    int nk2 = sparse ? std::min(4, pick_nk(kNk2, B, pl.nvec, sms)) : pick_nk(kNk2, B, pl.nvec, sms);
+    if (sms > 0) {  // segment sizes forced for tests and tuning (never above the workspace bound)
+      if (const char* e = std::getenv("DIPSD_SPEC_NK1"))
+        for (int v : kNk1) if (v == std::atoi(e)) nk1 = v;
+      if (const char* e = std::getenv("DIPSD_SPEC_NK2"))
+        for (int v : kNk2) if (v == std::atoi(e) && !(sparse && v > 4)) nk2 = v;
+    }
     const int nseg1 = ceil_div(pl.nvec, 32 * nk1), nseg2 = ceil_div(pl.nvec, 32 * nk2);
-    const long long items1 = static_cast<long long>(pl.sum_t + pl.sum_l) * nseg1;
+    const long long items1 = static_cast<long long>(rows) * nseg1;
     const long long items2 = static_cast<long long>(B) * nseg2;
     if (2 * nseg1 <= kMaxArrivals && nseg2 <= kMaxArrivals && items1 < (1ll << 31) && items2 < (1ll << 31)) {
       pl.nk1 = nk1; pl.nk2 = nk2;
@@ -481,6 +490,21 @@ size_t spec_ws_need(int B, const int* L, int V) {
   return need;
 }
 
+// Workspace of the sparse-payload path (16-byte aligned rows only).
+size_t spec_ws_need_sparse(int B, const int* L, int V) {
+  SpecPlan pl;
+  size_t need = 0;
+  if (V % 8 == 0) {
+    plan_spec(B, L, V, 2, true, 0, pl, true);
+    need = std::max(need, pl.ws_bytes);
+  }
+  if (V % 4 == 0) {
+    plan_spec(B, L, V, 4, true, 0, pl, true);
+    need = std::max(need, pl.ws_bytes);
+  }
+  return need;
+}
+
 template <typename T, int VEC, int CAP>
 int launch_spec_t(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s, bool pdl) {
   if (launch(spec_stats_generic_kernel<T, VEC, CAP>, dim3(pl.sum_t * pl.cl1), dim3(kSpecThreads), 0, s, pl.cl1,
@@ -492,37 +516,49 @@ int launch_spec_t(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s, 
   return DIPSD_OK;
 }
 
-template <typename T, int NK2, int CAP>
+template <typename T, int NK2, int CAP, bool SP>
 int launch_spec_sample_t(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s) {
-  return launch(spec_sample_kernel<T, NK2, CAP>, dim3(ceil_div(pl.n_items2, kRegWarps)), dim3(kRegThreads), 0, s,
-                1, true, p) == cudaSuccess ? DIPSD_OK : DIPSD_ERR_CUDA;
+  return launch(spec_sample_kernel<T, NK2, CAP, SP>, dim3(ceil_div(pl.n_items2, kRegWarps)), dim3(kRegThreads), 0,
+                s, 1, true, p) == cudaSuccess ? DIPSD_OK : DIPSD_ERR_CUDA;
 }
 
-template <typename T, int NK1, int CAP>
+template <typename T, int NK1, int CAP, bool SP>
 int launch_spec_reg_t(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s, bool pdl) {
-  if (launch(spec_stats_kernel<T, NK1, CAP>, dim3(ceil_div(pl.n_items1, kRegWarps)), dim3(kRegThreads), 0, s, 1,
+  if (launch(spec_stats_kernel<T, NK1, CAP, SP>, dim3(ceil_div(pl.n_items1, kRegWarps)), dim3(kRegThreads), 0, s, 1,
              pdl, p) != cudaSuccess)
     return DIPSD_ERR_CUDA;
-  switch (pl.nk2) {
-    case 8: return launch_spec_sample_t<T, 8, CAP>(pl, p, s);
-    case 4: return launch_spec_sample_t<T, 4, CAP>(pl, p, s);
-    default: return launch_spec_sample_t<T, 2, CAP>(pl, p, s);
+  if constexpr (SP) {  // the table's q of every element stays in registers: at most 4 vectors per lane
+    return pl.nk2 == 4 ? launch_spec_sample_t<T, 4, CAP, SP>(pl, p, s) : launch_spec_sample_t<T, 2, CAP, SP>(pl, p, s);
+  } else {
+    switch (pl.nk2) {
+      case 8: return launch_spec_sample_t<T, 8, CAP, SP>(pl, p, s);
+      case 4: return launch_spec_sample_t<T, 4, CAP, SP>(pl, p, s);
+      default: return launch_spec_sample_t<T, 2, CAP, SP>(pl, p, s);
+    }
   }
 }
 
-template <typename T, int CAP>
+template <typename T, int CAP, bool SP>
 int launch_spec_reg(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s, bool pdl) {
   switch (pl.nk1) {
-    case 16: return launch_spec_reg_t<T, 16, CAP>(pl, p, s, pdl);
-    case 8: return launch_spec_reg_t<T, 8, CAP>(pl, p, s, pdl);
-    default: return launch_spec_reg_t<T, 4, CAP>(pl, p, s, pdl);
+    case 16: return launch_spec_reg_t<T, 16, CAP, SP>(pl, p, s, pdl);
+    case 8: return launch_spec_reg_t<T, 8, CAP, SP>(pl, p, s, pdl);
+    default: return launch_spec_reg_t<T, 4, CAP, SP>(pl, p, s, pdl);
   }
 }
+
+// Sparse draft payload of one call (null: dense draft logits).
+struct SparseDraft {
+  const float* draft_logq = nullptr;
+  const int* topk_idx = nullptr;
+  const float* topk_q = nullptr;
+  int topk = 0;
+};
 
 template <int CAP>
 int run_spec_cap(const SpecPlan& pl, int dtype, const void* z, const void* w, const int* dt, const float* uni,
                  int* acc, int* offs, int* toks, float* probs, unsigned* status, uint8_t* region,
-                 cudaStream_t s, bool pdl) {
+                 cudaStream_t s, bool pdl, const SparseDraft& sd) {
   static thread_local SpecParams<CAP> p;
   std::memset(&p, 0, sizeof(p));
   p.z = z; p.w = w; p.draft_tokens = dt; p.uniforms = uni;
@@ -538,9 +574,18 @@ int run_spec_cap(const SpecPlan& pl, int dtype, const void* z, const void* w, co
   p.status = status;
   p.B = pl.B; p.V = pl.V; p.nvec = pl.nvec;
   for (int i = 0; i <= pl.B; ++i) { p.q_off[i] = pl.q_off[i]; p.l_off[i] = pl.l_off[i]; }
+  if (pl.sparse) {
+    if (!pl.nk1) return DIPSD_ERR_UNSUPPORTED;
+    p.draft_logq = sd.draft_logq;
+    p.topk_idx = sd.topk_idx;
+    p.topk_q = sd.topk_q;
+    p.topk = sd.topk;
+    return dtype == DIPSD_BF16 ? launch_spec_reg<__nv_bfloat16, CAP, true>(pl, p, s, pdl)
+                               : launch_spec_reg<float, CAP, true>(pl, p, s, pdl);
+  }
   if (pl.nk1)
-    return dtype == DIPSD_BF16 ? launch_spec_reg<__nv_bfloat16, CAP>(pl, p, s, pdl)
-                               : launch_spec_reg<float, CAP>(pl, p, s, pdl);
+    return dtype == DIPSD_BF16 ? launch_spec_reg<__nv_bfloat16, CAP, false>(pl, p, s, pdl)
+                               : launch_spec_reg<float, CAP, false>(pl, p, s, pdl);
   if (dtype == DIPSD_BF16)
     return pl.vec == 8 ? launch_spec_t<__nv_bfloat16, 8, CAP>(pl, p, s, pdl)
                        : launch_spec_t<__nv_bfloat16, 1, CAP>(pl, p, s, pdl);
@@ -549,10 +594,10 @@ int run_spec_cap(const SpecPlan& pl, int dtype, const void* z, const void* w, co
 
 int run_spec(const SpecPlan& pl, int dtype, const void* z, const void* w, const int* dt, const float* uni,
              int* acc, int* offs, int* toks, float* probs, unsigned* status, uint8_t* region, cudaStream_t s,
-             bool pdl) {
+             bool pdl, const SparseDraft& sd = SparseDraft{}) {
   if (pl.B <= kCapSmall)
-    return run_spec_cap<kCapSmall>(pl, dtype, z, w, dt, uni, acc, offs, toks, probs, status, region, s, pdl);
-  return run_spec_cap<kCapLarge>(pl, dtype, z, w, dt, uni, acc, offs, toks, probs, status, region, s, pdl);
+    return run_spec_cap<kCapSmall>(pl, dtype, z, w, dt, uni, acc, offs, toks, probs, status, region, s, pdl, sd);
+  return run_spec_cap<kCapLarge>(pl, dtype, z, w, dt, uni, acc, offs, toks, probs, status, region, s, pdl, sd);
 }
 
 int check_spec_buffers(int dtype, const void* z, const void* w, const int* dt, const float* uni, int* acc,
@@ -702,6 +747,49 @@ int dipsd_spec_verify(int B, const int* h_L, int V, int logit_dtype, const void*
   st = run_spec(pl, logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
                 d_out_offsets, d_out_tokens, d_draft_probs, reinterpret_cast<unsigned*>(ws), ws + kHeaderBytes,
                 static_cast<cudaStream_t>(stream), true);
+  return st != DIPSD_OK ? st : cuda_status();
+}
+
+size_t dipsd_spec_verify_sparse_workspace_size(int B, const int* h_L, int V) {
+  if (check_spec_users(B, h_L, V) != DIPSD_OK) return 0;
+  const size_t need = spec_ws_need_sparse(B, h_L, V);
+  return need ? kHeaderBytes + need : 0;
+}
+
+int dipsd_spec_verify_sparse(int B, const int* h_L, int V, int K, int logit_dtype, const void* d_target_logits,
+                             const int* d_draft_tokens, const float* d_draft_logq, const int* d_topk_idx,
+                             const float* d_topk_q, const float* d_uniforms, int* d_accept_len, int* d_out_offsets,
+                             int* d_out_tokens, float* d_draft_probs, void* d_workspace, size_t workspace_bytes,
+                             void* stream) {
+  int st = check_spec_users(B, h_L, V);
+  if (st != DIPSD_OK) return st;
+  if (K < 1 || K > kMaxTopK) return DIPSD_ERR_INVALID_ARG;
+  long long sum_l = 0;
+  for (int i = 0; i < B; ++i) sum_l += h_L[i];
+  bool vec_ok = false;
+  // (the draft-logits slot is checked with the target logits' pointer: the sparse path has none)
+  st = check_spec_buffers(logit_dtype, d_target_logits, d_target_logits, d_draft_tokens, d_uniforms, d_accept_len,
+                          d_out_offsets, d_out_tokens, d_draft_probs, static_cast<int>(sum_l), V, &vec_ok);
+  if (st != DIPSD_OK) return st;
+  if (sum_l > 0 && (!d_draft_logq || !d_topk_idx || !d_topk_q || !aligned(d_draft_logq, 4) ||
+                    !aligned(d_topk_idx, 4) || !aligned(d_topk_q, 4)))
+    return DIPSD_ERR_INVALID_ARG;
+  if (!vec_ok) return DIPSD_ERR_UNSUPPORTED;
+  st = check_workspace(d_workspace, workspace_bytes, kHeaderBytes + spec_ws_need_sparse(B, h_L, V));
+  if (st != DIPSD_OK) return st;
+  DeviceFacts f;
+  if (!device_facts(f)) return DIPSD_ERR_CUDA;
+  SpecPlan pl;
+  plan_spec(B, h_L, V, logit_dtype == DIPSD_BF16 ? 2 : 4, vec_ok, f.sms, pl, true);
+  SparseDraft sd;
+  sd.draft_logq = d_draft_logq;
+  sd.topk_idx = d_topk_idx;
+  sd.topk_q = d_topk_q;
+  sd.topk = K;
+  uint8_t* ws = static_cast<uint8_t*>(d_workspace);
+  st = run_spec(pl, logit_dtype, d_target_logits, nullptr, d_draft_tokens, d_uniforms, d_accept_len, d_out_offsets,
+                d_out_tokens, d_draft_probs, reinterpret_cast<unsigned*>(ws), ws + kHeaderBytes,
+                static_cast<cudaStream_t>(stream), true, sd);
   return st != DIPSD_OK ? st : cuda_status();
 }
 

@@ -11,6 +11,7 @@ constexpr int kSpecThreads = 256;
 constexpr int kSpecWarps = kSpecThreads / 32;
 constexpr int kMaxCluster = 8;
 constexpr unsigned kDevErrBadToken = 2u;
+constexpr int kMaxTopK = 64;  // sparse payload: table entries per draft row
 // Arrival counters of the register path, in 32-bit words: one per verify
 // position; then one 64-bit word per user for the decisions (arrivals in the
 // high half, acceptance bit t of position t in the low half); then one per
@@ -33,6 +34,12 @@ struct SpecParams {
   int* out_tokens;            // [sum T]
   unsigned* status;
   // register path only: segment partial sums and arrival counters
+  // sparse draft payload (spec_verify_sparse): per draft row, log q(d) and
+  // a table of topk (token, q) entries; q is 0 off the table
+  const float* draft_logq;  // [sum L]
+  const int* topk_idx;      // [sum L][topk]
+  const float* topk_q;      // [sum L][topk]
+  int topk;
   float4* part1;       // [n_items1] one per segment of every row
   float4* part2;       // [n_items2] one per segment of the sampled rows
   unsigned* counters;  // [kCounterWords], zero between calls

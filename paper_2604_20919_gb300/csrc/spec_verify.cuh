@@ -396,11 +396,106 @@ __device__ __forceinline__ void segment_totals(const uint4 (&rz)[NK], const uint
   if (!residual) tr = tp;
 }
 
+// segment_totals for a sparse draft table: q of each element from qx.
+template <typename T, int NK>
+__device__ __forceinline__ void segment_totals_table(const uint4 (&rz)[NK], const float (&qx)[NK][Vec16<T>::N],
+                                                     int nv, bool residual, const WRef& st, int lane, FF& tr,
+                                                     FF& tp) {
+  constexpr int N = Vec16<T>::N;
+  tr = FF{0.f, 0.f};
+  tp = FF{0.f, 0.f};
+#pragma unroll
+  for (int k = 0; k < NK; ++k) {
+    float sr = 0.f, sp = 0.f;
+    if (k < nv) {
+      float xz[N];
+      Vec16<T>::unpack(rz[k], xz);
+#pragma unroll
+      for (int e = 0; e < N; ++e) {
+        const float ez = ex2_ref(xz[e], st.cz);
+        sr = __fadd_rn(sr, residual && qx[k][e] > 0.f
+                               ? fmaxf(__fsub_rn(ez, __fmaf_rn(qx[k][e], st.khi, __fmul_rn(qx[k][e], st.klo))), 0.f)
+                               : ez);
+        sp = __fadd_rn(sp, ez);
+      }
+    }
+    const float gp = __shfl_sync(0xffffffffu, warp_scan_f32(sp, lane), 31);
+    tp = ff_add(tp, FF{gp, 0.f});
+    if (residual) {
+      const float gr = __shfl_sync(0xffffffffu, warp_scan_f32(sr, lane), 31);
+      tr = ff_add(tr, FF{gr, 0.f});
+    }
+  }
+  if (!residual) tr = tp;
+}
+
+// ------------------------------------------------------ sparse draft table
+// The draft row's table entries, two per lane (entry j in lane j % 32).
+__device__ __forceinline__ void load_table(const int* idx_row, const float* q_row, int K, int lane, int (&sidx)[2],
+                                           float (&sq)[2]) {
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int j = h * 32 + lane;
+    sidx[h] = j < K ? idx_row[j] : -1;
+    sq[h] = j < K ? q_row[j] : 0.f;
+  }
+}
+
+// q of every element of a lane's vectors vb + k * 32 + lane (k < nv) from
+// the table: 0 off the table.  Warp-uniform: each lane tests its two entries
+// against the segment's token range, and only the entries that fall inside
+// (a ballot) go round by shuffle.
+template <int NK, int N>
+__device__ __forceinline__ void table_q(const int (&sidx)[2], const float (&sq)[2], int K, int V, int vb, int lane,
+                                        int nv, float (&qx)[NK][N], unsigned* status) {
+#pragma unroll
+  for (int k = 0; k < NK; ++k)
+#pragma unroll
+    for (int e = 0; e < N; ++e) qx[k][e] = 0.f;
+  const int lo = vb * N, hi = (vb + 32 * NK) * N;  // tokens of the segment
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int j = h * 32 + lane;
+    if (j < K && (sidx[h] < 0 || sidx[h] >= V)) atomicOr(status, kDevErrBadToken);
+    unsigned hits = __ballot_sync(0xffffffffu, j < K && sidx[h] >= lo && sidx[h] < hi && sidx[h] < V);
+    while (hits) {
+      const int src = __ffs(hits) - 1;
+      hits &= hits - 1;
+      const int idx = __shfl_sync(0xffffffffu, sidx[h], src);
+      const float qv = __shfl_sync(0xffffffffu, sq[h], src);
+      const int dv = idx / N - vb - lane;
+      if (dv < 0 || (dv & 31) != 0 || (dv >> 5) >= nv) continue;
+      const int kk = dv >> 5, ee = idx % N;
+#pragma unroll
+      for (int k = 0; k < NK; ++k)
+#pragma unroll
+        for (int e = 0; e < N; ++e)
+          if (k == kk && e == ee) qx[k][e] = qv;
+    }
+  }
+}
+
+// Sampling weights of one vector from a sparse table: max(0, p - q) up to
+// the factor 1/sz (e_z - q sz, sz as khi + klo) where q > 0, else p's e_z
+// (residual), or p's e_z.  Same rounding wherever it is evaluated.
+template <typename T>
+__device__ __forceinline__ void vec_weights_table(const uint4& rz, const float (&qx)[Vec16<T>::N], bool residual,
+                                                  int cz, float khi, float klo, float (&wt)[Vec16<T>::N]) {
+  constexpr int N = Vec16<T>::N;
+  float xz[N];
+  Vec16<T>::unpack(rz, xz);
+#pragma unroll
+  for (int e = 0; e < N; ++e) {
+    const float ez = ex2_ref(xz[e], cz);
+    wt[e] = residual && qx[e] > 0.f ? fmaxf(__fsub_rn(ez, __fmaf_rn(qx[e], khi, __fmul_rn(qx[e], klo))), 0.f) : ez;
+  }
+}
+
 // ----------------------------------------------------- position decision
 // Run by the warp that delivered the last segment of position q0 + t of user
 // ui: row sums, p_t(d), q_t(d), the acceptance decision; the user's last
 // decided position also writes a_i.
-template <int CAP>
+template <int CAP, bool SP>
 __device__ __forceinline__ void decide_position(const SpecParams<CAP>& p, int ui, int t, int lane) {
   const int q0 = p.q_off[ui];
   const int Li = p.q_off[ui + 1] - q0 - 1;
@@ -410,21 +505,22 @@ __device__ __forceinline__ void decide_position(const SpecParams<CAP>& p, int ui
   const float4* pw = p.part1 + static_cast<size_t>(p.sum_t + l) * p.nseg1;
   // every load first: the draft token's logits, left by the rows' first
   // segments (NaN: d outside [0, V)), and both rows' segment partials
-  float zd = 0.f, wd = 0.f;
+  float zd = 0.f, wd = 0.f, logq = 0.f;
   if (has_q && lane == 0) {
     zd = __ldcg(&pz->w);
-    wd = __ldcg(&pw->w);
+    if constexpr (SP) logq = p.draft_logq[l];
+    else wd = __ldcg(&pw->w);
   }
   RefSum az{kEmptyRef, FF{0.f, 0.f}}, aw{kEmptyRef, FF{0.f, 0.f}};
 #pragma unroll 2
   for (int sg = lane; sg < p.nseg1; sg += 32) {
     const float4 vz = __ldcg(pz + sg);
-    const float4 vw = has_q ? __ldcg(pw + sg) : make_float4(__int_as_float(kEmptyRef), 0.f, 0.f, 0.f);
+    const float4 vw = has_q && !SP ? __ldcg(pw + sg) : make_float4(__int_as_float(kEmptyRef), 0.f, 0.f, 0.f);
     az = refsum_add(az, RefSum{__float_as_int(vz.x), FF{vz.y, vz.z}});
     aw = refsum_add(aw, RefSum{__float_as_int(vw.x), FF{vw.y, vw.z}});
   }
   az = warp_refsum(az);
-  if (has_q) aw = warp_refsum(aw);
+  if (has_q && !SP) aw = warp_refsum(aw);
   if (lane == 0) {
     p.counters[n] = 0u;
     SpecStat st;
@@ -435,7 +531,22 @@ __device__ __forceinline__ void decide_position(const SpecParams<CAP>& p, int ui
     st.khi = st.klo = 0.f;
     float pd = 0.f, qd = 0.f;
     unsigned char flag = 0;
-    if (has_q) {
+    if (has_q && SP) {
+      // sparse payload: q(d) is given; the residual scales q by sz, kept as
+      // a float-float pair
+      st.khi = az.s.hi;
+      st.klo = az.s.lo;
+      if (zd == zd) {
+        const float ez = ex2_ref(zd, st.cz);
+        const double q_d = exp(static_cast<double>(logq));
+        pd = ez * (1.f / static_cast<float>(st.sz));
+        qd = static_cast<float>(q_d);
+        // u * q(d) < p(d) = ez / sz, i.e. u * q(d) * sz < ez
+        flag = static_cast<double>(p.uniforms[2 * n]) * q_d * st.sz < static_cast<double>(ez) ? 1 : 0;
+      } else {
+        atomicOr(p.status, kDevErrBadToken);
+      }
+    } else if (has_q) {
       st.sw = static_cast<double>(aw.s.hi) + static_cast<double>(aw.s.lo);
       st.cw = aw.c;
       // sz / sw in float-float: q1 = zh / wh, then the remainder's quotient
@@ -472,7 +583,7 @@ __device__ __forceinline__ void decide_position(const SpecParams<CAP>& p, int ui
 }
 
 // ------------------------------------------------------------------ pass 1
-template <typename T, int NK, int CAP>
+template <typename T, int NK, int CAP, bool SP>
 __global__ void __launch_bounds__(kRegThreads, 2)
 spec_stats_kernel(const __grid_constant__ SpecParams<CAP> p) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -482,7 +593,7 @@ spec_stats_kernel(const __grid_constant__ SpecParams<CAP> p) {
   if (item >= p.n_items1) return;
   const int row = item / p.nseg1;
   const int s = item - row * p.nseg1;
-  const bool is_w = row >= p.sum_t;  // rows: every z_t, then every w_t
+  const bool is_w = !SP && row >= p.sum_t;  // rows: every z_t, then every w_t (none when sparse)
   const int ui = is_w ? spec_find_user<CAP>(p.l_off, p.B, row - p.sum_t) : spec_find_user<CAP>(p.q_off, p.B, row);
   const int q0 = p.q_off[ui];
   const int Li = p.q_off[ui + 1] - q0 - 1;
@@ -521,16 +632,17 @@ spec_stats_kernel(const __grid_constant__ SpecParams<CAP> p) {
   }
   __syncwarp();
   cnt = __shfl_sync(0xffffffffu, cnt, 0);
-  if (cnt != static_cast<unsigned>(p.nseg1 * (has_q ? 2 : 1))) return;
-  decide_position<CAP>(p, ui, t, lane);
+  if (cnt != static_cast<unsigned>(p.nseg1 * (has_q && !SP ? 2 : 1))) return;
+  decide_position<CAP, SP>(p, ui, t, lane);
 }
 
 // ------------------------------------------------------------------ pass 2
 // Run by the warp that delivered the last segment of user ui: packed output
 // offset, accepted drafts, then the inverse-CDF descent to the emitted token.
-template <typename T, int NK, int CAP>
+template <typename T, int NK, int CAP, bool SP>
 __device__ __forceinline__ void descend(const SpecParams<CAP>& p, int ui, int a, bool residual, const WRef& st,
-                                        const T* zrow, const T* wrow, int lane) {
+                                        const T* zrow, const T* wrow, const int (&sidx)[2], const float (&sq)[2],
+                                        int lane) {
   constexpr int N = Vec16<T>::N;
   const int q0 = p.q_off[ui], l0 = p.l_off[ui];
   const int n = q0 + a;
@@ -634,14 +746,24 @@ __device__ __forceinline__ void descend(const SpecParams<CAP>& p, int ui, int a,
     const int nv = lane_vectors(p.nvec, vb, lane, NK);
     uint4 rz[NK], rw[NK];
     load_segment<NK>(zrow, vb, lane, nv, rz);
-    load_segment<NK>(wrow, vb, lane, residual ? nv : 0, rw);
+    load_segment<NK>(wrow, vb, lane, residual && !SP ? nv : 0, rw);
+    float qx[NK][N];
+    if constexpr (SP) {
+      if (residual) table_q<NK, N>(sidx, sq, p.topk, p.V, vb, lane, nv, qx, p.status);
+      else
+#pragma unroll
+        for (int k = 0; k < NK; ++k)
+#pragma unroll
+          for (int e = 0; e < N; ++e) qx[k][e] = 0.f;
+    }
     float vs[NK], gin[NK];
 #pragma unroll
     for (int k = 0; k < NK; ++k) {
       vs[k] = 0.f;
       if (k < nv) {
         float wt[N];
-        vec_weights<T>(rz[k], rw[k], mode == 0, st.cz, st.cw, st.khi, st.klo, wt);
+        if constexpr (SP) vec_weights_table<T>(rz[k], qx[k], mode == 0, st.cz, st.khi, st.klo, wt);
+        else vec_weights<T>(rz[k], rw[k], mode == 0, st.cz, st.cw, st.khi, st.klo, wt);
         vs[k] = vec_sum<N>(wt);
       }
       gin[k] = warp_scan_f32(vs[k], lane);
@@ -666,6 +788,9 @@ __device__ __forceinline__ void descend(const SpecParams<CAP>& p, int ui, int a,
     // level 3: the lane of group kk, then the token inside its vector
     float ik = 0.f, vk = 0.f;
     uint4 mz = rz[0], mw = rw[0];
+    float mq[N];
+#pragma unroll
+    for (int e = 0; e < N; ++e) mq[e] = 0.f;
 #pragma unroll
     for (int k = 0; k < NK; ++k)
       if (k == kk) {
@@ -673,6 +798,9 @@ __device__ __forceinline__ void descend(const SpecParams<CAP>& p, int ui, int a,
         vk = vs[k];
         mz = rz[k];
         mw = rw[k];
+        if constexpr (SP)
+#pragma unroll
+          for (int e = 0; e < N; ++e) mq[e] = qx[k][e];
       }
     int ln2 = -1;
     if (!last) {
@@ -691,7 +819,10 @@ __device__ __forceinline__ void descend(const SpecParams<CAP>& p, int ui, int a,
       float wt[N];
 #pragma unroll
       for (int e = 0; e < N; ++e) wt[e] = 0.f;
-      if (kk < nv) vec_weights<T>(mz, mw, mode == 0, st.cz, st.cw, st.khi, st.klo, wt);
+      if (kk < nv) {
+        if constexpr (SP) vec_weights_table<T>(mz, mq, mode == 0, st.cz, st.khi, st.klo, wt);
+        else vec_weights<T>(mz, mw, mode == 0, st.cz, st.cw, st.khi, st.klo, wt);
+      }
       int es = -1;
       if (!last) {
         float cum = 0.f;
@@ -714,7 +845,7 @@ __device__ __forceinline__ void descend(const SpecParams<CAP>& p, int ui, int a,
   if (lane == 0) p.out_tokens[off + a] = 0;  // no mass at all: every logit -inf
 }
 
-template <typename T, int NK, int CAP>
+template <typename T, int NK, int CAP, bool SP>
 __global__ void __launch_bounds__(kRegThreads, 2)
 spec_sample_kernel(const __grid_constant__ SpecParams<CAP> p) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -739,14 +870,32 @@ spec_sample_kernel(const __grid_constant__ SpecParams<CAP> p) {
   st.khi = __int_as_float(__shfl_sync(0xffffffffu, ref4.z, a));
   st.klo = __int_as_float(__shfl_sync(0xffffffffu, ref4.w, a));
   const T* zrow = static_cast<const T*>(p.z) + static_cast<size_t>(n) * p.V;
-  const T* wrow = residual ? static_cast<const T*>(p.w) + static_cast<size_t>(l0 + a) * p.V : zrow;
+  const T* wrow = residual && !SP ? static_cast<const T*>(p.w) + static_cast<size_t>(l0 + a) * p.V : zrow;
   const int vb = s * (32 * NK);
   const int nv = lane_vectors(p.nvec, vb, lane, NK);
   uint4 rz[NK], rw[NK];
   load_segment<NK>(zrow, vb, lane, nv, rz);
-  load_segment<NK>(wrow, vb, lane, residual ? nv : 0, rw);
+  load_segment<NK>(wrow, vb, lane, residual && !SP ? nv : 0, rw);
+  int sidx[2] = {-1, -1};
+  float sq[2] = {0.f, 0.f};
   FF R, P;
-  segment_totals<T, NK>(rz, rw, nv, residual, st, lane, R, P);
+  if constexpr (SP) {
+    constexpr int N = Vec16<T>::N;
+    float qx[NK][N];
+    if (residual) {
+      load_table(p.topk_idx + static_cast<size_t>(l0 + a) * p.topk, p.topk_q + static_cast<size_t>(l0 + a) * p.topk,
+                 p.topk, lane, sidx, sq);
+      table_q<NK, N>(sidx, sq, p.topk, p.V, vb, lane, nv, qx, p.status);
+    } else {
+#pragma unroll
+      for (int k = 0; k < NK; ++k)
+#pragma unroll
+        for (int e = 0; e < N; ++e) qx[k][e] = 0.f;
+    }
+    segment_totals_table<T, NK>(rz, qx, nv, residual, st, lane, R, P);
+  } else {
+    segment_totals<T, NK>(rz, rw, nv, residual, st, lane, R, P);
+  }
   unsigned cnt = 0;
   if (lane == 31) {
     p.part2[item] = make_float4(R.hi, R.lo, P.hi, P.lo);
@@ -755,7 +904,7 @@ spec_sample_kernel(const __grid_constant__ SpecParams<CAP> p) {
   __syncwarp();
   cnt = __shfl_sync(0xffffffffu, cnt, 31);
   if (cnt != static_cast<unsigned>(p.nseg2)) return;
-  descend<T, NK, CAP>(p, ui, a, residual, st, zrow, wrow, lane);
+  descend<T, NK, CAP, SP>(p, ui, a, residual, st, zrow, wrow, sidx, sq, lane);
 }
 
 }  // namespace dipsd

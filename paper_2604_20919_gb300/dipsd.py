@@ -34,6 +34,7 @@ EXPORTS = (
     "dipsd_spec_verify_workspace_size", "dipsd_spec_verify",
     "dipsd_verify_batch_workspace_size", "dipsd_verify_batch", "dipsd_spec_verify_noalloc",
     "dipsd_verify_attention_append", "dipsd_verify_batch_append",
+    "dipsd_spec_verify_sparse_workspace_size", "dipsd_spec_verify_sparse",
 )
 NOALLOC_MAX_POSITIONS = 4096
 
@@ -84,6 +85,11 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.dipsd_verify_batch_append.argtypes = [_i, _i32p, _i, _i32p, _i32p, _vp, _vp, _vp, _vp, _vp, _i, _vp, _i,
                                               _i, _i, _i, ctypes.c_float, _vp, _i, _i, _vp, _vp, _vp, _vp, _vp,
                                               _vp, _vp, _vp, _vp, _sz, _vp]
+    lib.dipsd_spec_verify_sparse_workspace_size.restype = _sz
+    lib.dipsd_spec_verify_sparse_workspace_size.argtypes = [_i, _i32p, _i]
+    lib.dipsd_spec_verify_sparse.restype = _i
+    lib.dipsd_spec_verify_sparse.argtypes = [_i, _i32p, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                             _vp, _sz, _vp]
     lib.dipsd_spec_verify_noalloc.restype = _i
     lib.dipsd_spec_verify_noalloc.argtypes = [_i, _i32p, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]
     _lib = lib
@@ -250,6 +256,43 @@ def dipsd_spec_verify(L, target_logits, draft_logits, draft_tokens, uniforms, ou
                                _dptr(probs, "draft_probs", torch.float32), _dptr(ws, "workspace"), ws.numel(),
                                _stream(stream))
     _check(st, "dipsd_spec_verify")
+    return acc, offs, toks, probs
+
+
+def dipsd_spec_verify_sparse_workspace_size(L, V: int) -> int:
+    a, pa = _host_i32(L)
+    return int(load().dipsd_spec_verify_sparse_workspace_size(len(a), pa, V))
+
+
+def dipsd_spec_verify_sparse(L, target_logits, draft_tokens, draft_logq, topk_idx, topk_q, uniforms, outputs=None,
+                             ws=None, stream=None):
+    """Speculative verification from a sparse draft payload; returns
+    (accept_len, out_offsets, out_tokens, draft_probs)."""
+    lib = load()
+    a, pa = _host_i32(L)
+    sum_t, sum_l = int((a + 1).sum()), int(a.sum())
+    V = target_logits.shape[1]
+    K = int(topk_idx.shape[1]) if topk_idx.dim() == 2 else 0
+    if target_logits.shape[0] != sum_t or tuple(uniforms.shape) != (sum_t, 2):
+        raise ValueError("target_logits / uniforms do not match the draft lengths")
+    if (draft_tokens.numel() != sum_l or draft_logq.numel() != sum_l or tuple(topk_idx.shape) != (sum_l, K)
+            or tuple(topk_q.shape) != (sum_l, K)):
+        raise ValueError("draft tokens / log-probabilities / table do not match the draft lengths")
+    acc, offs, toks, probs = outputs if outputs is not None else spec_outputs(a, target_logits.device)
+    if ws is None:
+        ws = workspace(dipsd_spec_verify_sparse_workspace_size(a, V), target_logits.device)
+    st = lib.dipsd_spec_verify_sparse(len(a), pa, V, max(K, 1), _logit_dtype(target_logits),
+                                      _dptr(target_logits, "target_logits"),
+                                      _dptr(draft_tokens, "draft_tokens", torch.int32) if sum_l else 0,
+                                      _dptr(draft_logq, "draft_logq", torch.float32) if sum_l else 0,
+                                      _dptr(topk_idx, "topk_idx", torch.int32) if sum_l else 0,
+                                      _dptr(topk_q, "topk_q", torch.float32) if sum_l else 0,
+                                      _dptr(uniforms, "uniforms", torch.float32),
+                                      _dptr(acc, "accept_len", torch.int32), _dptr(offs, "out_offsets", torch.int32),
+                                      _dptr(toks, "out_tokens", torch.int32),
+                                      _dptr(probs, "draft_probs", torch.float32), _dptr(ws, "workspace"), ws.numel(),
+                                      _stream(stream))
+    _check(st, "dipsd_spec_verify_sparse")
     return acc, offs, toks, probs
 
 

@@ -19,7 +19,7 @@ import pytest
 import scipy.special
 import scipy.stats
 
-from oracle import inverse_cdf, softmax, spec_verify
+from oracle import inverse_cdf, softmax, spec_verify, spec_verify_sparse
 from oracle.spec_verify import residual
 
 
@@ -249,3 +249,105 @@ def test_truncation_and_packing_invariants():
         assert not acc[qo + L[i]]  # bonus position carries no test
         qo += T[i]
         lo += L[i]
+
+
+# ---------------------------------------------------------------------------
+# sparse draft payload (spec_verify_sparse)
+# ---------------------------------------------------------------------------
+
+def _sparse_table(q):
+    """(topk_idx, topk_q) rows of a dense draft distribution's support, padded
+    with zero-probability entries on tokens outside the support."""
+    K = int(max((q > 0).sum(axis=1).max(), 1)) if len(q) else 1
+    idx = np.zeros((len(q), K), dtype=np.int64)
+    val = np.zeros((len(q), K))
+    for r in range(len(q)):
+        sup = np.flatnonzero(q[r] > 0)
+        off = [x for x in range(q.shape[1]) if x not in set(sup)]
+        pad = off[:K - len(sup)]
+        idx[r] = np.concatenate([sup, pad]).astype(np.int64)
+        val[r, :len(sup)] = q[r, sup]
+    return idx, val
+
+
+def _enumerated_law_sparse(zl, q, L):
+    """P(emitted sequence) by enumeration through spec_verify_sparse, q dense with zeros."""
+    V = zl.shape[1]
+    p = scipy.special.softmax(zl, axis=-1)
+    acc_cells = [_cells(np.minimum(1.0, np.divide(p[t], q[t], out=np.ones(V), where=q[t] > 0))) for t in range(L)]
+    res_cells = []
+    for t in range(L + 1):
+        pts = [np.cumsum(p[t])]
+        if t < L:
+            r = np.maximum(p[t] - q[t], 0)
+            if r.sum() > 0:
+                pts.append(np.cumsum(r) / r.sum())
+        res_cells.append(_cells(np.concatenate(pts)))
+    idx, val = _sparse_table(q)
+    rows_d, rows_u, weights = [], [], []
+    for drafts in itertools.product(range(V), repeat=L):
+        w_d = np.prod([q[t, drafts[t]] for t in range(L)]) if L else 1.0
+        if w_d == 0:
+            continue
+        for acc in itertools.product(*[range(len(c[0])) for c in acc_cells]):
+            w_a = np.prod([acc_cells[t][1][acc[t]] for t in range(L)]) if L else 1.0
+            for res in itertools.product(*[range(len(c[0])) for c in res_cells]):
+                w_r = np.prod([res_cells[t][1][res[t]] for t in range(L + 1)])
+                u = np.zeros((L + 1, 2))
+                for t in range(L):
+                    u[t, 0] = acc_cells[t][0][acc[t]]
+                for t in range(L + 1):
+                    u[t, 1] = res_cells[t][0][res[t]]
+                rows_d.append(drafts)
+                rows_u.append(u)
+                weights.append(w_d * w_a * w_r)
+    n = len(weights)
+    d = np.array(rows_d, dtype=np.int64).reshape(-1)
+    logq = np.log(np.tile(q, (n, 1))[np.arange(n * L), d]) if L else np.zeros(0)
+    out = spec_verify_sparse(np.full(n, L), np.tile(zl, (n, 1)), d, logq, np.tile(idx, (n, 1)),
+                             np.tile(val, (n, 1)), np.concatenate(rows_u))
+    law = {}
+    offs = out["out_offsets"]
+    for i in range(n):
+        seq = tuple(int(x) for x in out["out_tokens"][offs[i]:offs[i + 1]])
+        law[seq] = law.get(seq, 0.0) + weights[i]
+    return law, p
+
+
+@pytest.mark.parametrize("V,L,K,seed", [(4, 1, 2, 11), (3, 2, 1, 12), (4, 2, 3, 13), (5, 1, 5, 14)])
+def test_sparse_output_law_matches_closed_form(V, L, K, seed):
+    """A draft distribution on K of V tokens: the enumerated output law equals
+    prod_t min(p_t, q_t) x (residual or p), and the first token is p_0."""
+    rng = np.random.default_rng(seed)
+    zl = rng.normal(0, 1.5, size=(L + 1, V))
+    q = np.zeros((L, V))
+    for t in range(L):
+        sup = rng.choice(V, size=K, replace=False)
+        q[t, sup] = rng.dirichlet(np.ones(K))
+    law, p = _enumerated_law_sparse(zl, q, L)
+    ref = _closed_form_law(p, q, L)
+    assert set(k for k, v in law.items() if v > 1e-15) == set(ref)
+    for k, v in ref.items():
+        assert abs(law[k] - v) < 1e-12, (k, law[k], v)
+    first = np.zeros(V)
+    for k, v in law.items():
+        first[k[0]] += v
+    np.testing.assert_allclose(first, p[0], atol=1e-12)
+
+
+def test_sparse_with_full_support_equals_dense():
+    """K = V, q = softmax(w), logq(d) = log q(d): spec_verify_sparse == spec_verify."""
+    rng = np.random.default_rng(15)
+    L = np.array([3, 0, 5, 2])
+    V = 40
+    z = rng.normal(0, 2, size=(int((L + 1).sum()), V))
+    w = z[np.concatenate([np.arange(o, o + l) for o, l in zip(np.concatenate([[0], np.cumsum(L + 1)[:-1]]), L)])]
+    w = w + rng.normal(0, 0.7, size=w.shape)
+    q = scipy.special.softmax(w, axis=-1)
+    d = np.array([rng.choice(V, p=q[r]) for r in range(len(q))])
+    u = rng.random((len(z), 2))
+    dense = spec_verify(L, z, w, d, u)
+    idx = np.tile(np.arange(V), (len(q), 1))
+    sparse = spec_verify_sparse(L, z, d, np.log(q[np.arange(len(q)), d]), idx, q, u)
+    for key in ("accept_len", "out_offsets", "out_tokens", "accepted"):
+        assert np.array_equal(dense[key], sparse[key]), key

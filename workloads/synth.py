@@ -187,6 +187,45 @@ def make_spec_inputs(rng, L, user_ids, V, logit_std, noise_sigma, logit_dtype, s
     return zt, wt, torch.from_numpy(d), torch.from_numpy(uni)
 
 
+@dataclass
+class SparseDraft:
+    """A sparse draft payload: per draft row, K support tokens with their draft
+    probabilities, the draft token drawn from them, and its log-probability."""
+    topk_idx: torch.Tensor     # int32 [sum L, K], distinct tokens
+    topk_q: torch.Tensor       # fp32 [sum L, K], >= 0, summing to ~1 per row
+    draft_tokens: torch.Tensor  # int32 [sum L]
+    draft_logq: torch.Tensor   # fp32 [sum L]: log of the stored q of the draft token
+
+
+def make_sparse_draft(b: "Batch", K: int, seed: int = 0, rank_noise: float = 1.0, device="cpu") -> SparseDraft:
+    """The device's side of a sparse payload for batch b: per draft row the K
+    tokens ranked highest by (stored target logit + Gaussian noise), Dirichlet(1)
+    probabilities sorted so the best-ranked token gets the largest, and a draft
+    token drawn from them (numpy's categorical sampler, the device's job)."""
+    rng = np.random.default_rng([seed, 77])
+    z = b.target_logits.double().cpu().numpy()
+    qo, lo = offsets(b.T), offsets(b.L)
+    sL = int(b.L.sum())
+    idx = np.zeros((sL, K), dtype=np.int32)
+    qv = np.zeros((sL, K), dtype=np.float32)
+    d = np.zeros(sL, dtype=np.int32)
+    logq = np.zeros(sL, dtype=np.float32)
+    for i in range(b.B):
+        for t in range(int(b.L[i])):
+            r = lo[i] + t
+            score = z[qo[i] + t] + rng.normal(0.0, rank_noise, size=z.shape[1])
+            top = np.argpartition(-score, K - 1)[:K]
+            top = top[np.argsort(-score[top])]
+            idx[r] = top
+            qv[r] = np.sort(rng.dirichlet(np.ones(K)))[::-1].astype(np.float32)
+            pr = qv[r].astype(np.float64)
+            j = int(rng.choice(K, p=pr / pr.sum()))
+            d[r] = top[j]
+            logq[r] = np.float32(np.log(np.float64(qv[r, j])))
+    return SparseDraft(topk_idx=torch.from_numpy(idx).to(device), topk_q=torch.from_numpy(qv).to(device),
+                       draft_tokens=torch.from_numpy(d).to(device), draft_logq=torch.from_numpy(logq).to(device))
+
+
 def make_batch(L, ctx, *, Hq, Hkv, D, V, logit_std=1.0, noise_sigma=1.0,
                logit_dtype="bf16", seed=0, device="cpu", kv_device=None,
                alpha=None, spare_pages=3, user_ids=None, spec_only=False) -> Batch:
