@@ -13,7 +13,6 @@
 
 namespace dipsd {
 
-constexpr int kAttnTile = 64;  // KV tokens per pipeline stage (4 pages)
 constexpr unsigned kDevErrBadBlock = 4u;  // an appended row's page id outside [0, num_blocks)
 
 struct AttnUser {
@@ -23,7 +22,7 @@ struct AttnUser {
   int kv_len;     // C_i + T
   int bt_row;     // block-table row of the user
   int nsplit;     // KV splits
-  int split_len;  // KV tokens per split (multiple of kAttnTile)
+  int split_len;  // KV tokens per split (a whole number of kernel tiles)
   int n_rb;       // row blocks
 };
 

@@ -6,21 +6,28 @@
 // pass), so each K/V byte brought on chip serves every row.
 //
 // Roles (6 warps):
-//   warp 0      TMA producer into a ring of kStages 64-token K tiles and a
-//               ring of as many V tiles (128-byte swizzle).  K: one box per
+//   warp 0      TMA producer into a ring of kStages 128-token K tiles and
+//               a ring of as many V tiles (128-byte swizzle).  K: one box per
 //               page and 64-column half (2 KB), stored half after half, so a
-//               half is 64 rows at the uniform 1024-byte stride one N=64
+//               half is 128 rows at the uniform 1024-byte stride one N=128
 //               product needs.  V: one box per page (4 KB at D = 128, both
 //               halves through a 5-D tensor map whose third dimension steps
 //               128 bytes), stored page after page.  K and V stages are
 //               released separately: K once its Q K^T has run, V after its
 //               P V.  Page ids are fetched 32 at a time, one per lane, a
-//               group ahead.
+//               group ahead; pages past the user's end are requested at an
+//               out-of-range block, which TMA fills with zeros without
+//               reading memory.
 //   warp 1      allocates TMEM; one thread issues tcgen05.mma as operands
 //               become ready (no fixed order between the two products):
-//                 S[b] = Q K^T      (A = Q from tensor memory, M=128, N=64)
+//                 S[b] = Q K^T      (A = Q from tensor memory, M=128, N=128)
 //                 O   += P[b] V     (A = P from tensor memory; a 16-key step
-//                                    is one page of V; two N=64 halves)
+//                                    is one page of V, N = D: the
+//                                    descriptor's leading offset steps to
+//                                    the page's second 64-column half)
+//               A tile costs 16 MMAs and 4 commits whatever D is; the
+//               issuing thread, not the tensor core, is what bounds the
+//               tile rate, so tiles are as long as the rings allow.
 //   warps 2..5  one query row per thread (TMEM lane = row): put the Q row
 //               in TMEM, then per tile load S[b] with
 //               tcgen05.ld, causal mask, online softmax in log2 units with a
@@ -38,8 +45,8 @@
 // block and head run as one thread-block cluster: the other ranks push their
 // rows into rank 0's drained rings through distributed shared memory and
 // rank 0 merges them with its own O straight from TMEM.
-// TMEM columns: S/P double buffer [0,64) [64,128), O [128, 128+D), Q [256,
-// 256 + D/2).  Shared memory holds only the two rings (Q and P live in
+// TMEM columns: S/P double buffer [0,128) [128,256), O [256, 256+D), Q
+// [384, 384 + D/2).  Shared memory holds only the two rings (Q and P live in
 // tensor memory, so no product re-reads an operand from shared memory every
 // tile), which leaves room for kStages tiles of K and of V in flight.
 #pragma once
@@ -50,22 +57,29 @@
 namespace dipsd {
 
 constexpr int kTcThreads = 192;
-constexpr int kTcTile = 64;                // keys per tile
+constexpr int kTcTile = 128;               // keys per tile (8 pages)
 constexpr uint32_t kTmemCols = 512;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 
 template <int D>
 struct TcSmem {
   static constexpr int kHalves = D / 64;
-  static constexpr int kStages = D == 128 ? 7 : 12;
+  static constexpr int kStages = D == 128 ? 3 : 7;
   static constexpr int kPageBytes = kHalves * kPage * 128;           // V: [half][16 rows][128 B]
-  static constexpr int kTileBytes = (kTcTile / kPage) * kPageBytes;  // 64 keys x D bf16 (K or V)
+  static constexpr int kTileBytes = (kTcTile / kPage) * kPageBytes;  // 128 keys x D bf16 (K or V)
   static constexpr int kKOff = 0;
   static constexpr int kVOff = kKOff + kStages * kTileBytes;
   static constexpr int kBarOff = kVOff + kStages * kTileBytes;
   static constexpr int kBytes = kBarOff + 1024;  // barriers (6 kStages + 8) and the TMEM slot
   static constexpr int kAlloc = kBytes + 1024;  // slack for 1024-byte alignment
+  // cluster merge: the other ranks' (m, l, O) rows land in rank 0's drained
+  // rings, up to kMaxCluster - 1 of them
+  static constexpr int kMaxCluster = D == 128 ? 3 : 6;
+  static constexpr int kSlotBytes = 128 * 8 + 128 * D * 4;
 };
+static_assert((TcSmem<128>::kMaxCluster - 1) * TcSmem<128>::kSlotBytes <= TcSmem<128>::kBarOff, "exchange fits");
+static_assert((TcSmem<64>::kMaxCluster - 1) * TcSmem<64>::kSlotBytes <= TcSmem<64>::kBarOff, "exchange fits");
+static_assert(TcSmem<128>::kAlloc <= 232448 && TcSmem<64>::kAlloc <= 232448, "shared memory per CTA");
 constexpr int kTcStages = TcSmem<128>::kStages;
 
 // tm_k: 4-D {64 columns, 16 rows, heads, blocks}, one 64-column half of a
@@ -110,10 +124,12 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
   const int kv_begin = split * U.split_len;
   const int kv_end = min(kv_begin + U.split_len, U.kv_len);
   const int ntiles = max(0, (kv_end - kv_begin + kTcTile - 1) / kTcTile);  // 0: an empty split
-  // tile j holds new (appended) rows: keys [max(key0, C_i), min(key0 + 64, kv_len))
+  // Splits start on a page; a split's last tile may run past kv_end into the
+  // next split's keys, which are masked and never loaded.
+  // tile j holds new (appended) rows: keys [max(key0, C_i), min(key0 + 128, kv_end))
   auto patched = [&](int j) {
     const int key0 = kv_begin + j * kTcTile;
-    return p.new_k != nullptr && max(key0, U.ctx) < min(key0 + kTcTile, U.kv_len);
+    return p.new_k != nullptr && max(key0, U.ctx) < min(key0 + kTcTile, kv_end);
   };
 
   const int warp = threadIdx.x >> 5;
@@ -150,7 +166,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t tS0 = tmem, tO = tmem + 128, tQ = tmem + 256;
+  const uint32_t tS0 = tmem, tO = tmem + 2 * kTcTile, tQ = tmem + 384;
   float fin_m = -INFINITY, fin_l = 0.f;  // softmax threads: row state after the last tile
   bool fin_ok = false;
   pdl_wait_prior_grid();
@@ -161,13 +177,14 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
     // Page ids come from the block table 32 at a time (one per lane, one
     // group of 8 tiles ahead) so no TMA waits on a dependent global load.
     const int* bt = p.block_table + static_cast<size_t>(U.bt_row) * p.max_blocks;
-    const int n_pages = (U.kv_len + kPage - 1) / kPage;
+    const int n_pages = (kv_end + kPage - 1) / kPage;  // pages of this split end here
     const int page_base = kv_begin / kPage;
     auto fetch = [&](int group) {
       const int page = page_base + group * 32 + lane;
-      return page < n_pages ? __ldg(bt + page) : 0;
+      return page < n_pages ? __ldg(bt + page) : p.num_blocks;  // past the end: zero fill
     };
     constexpr int kPages = kTcTile / kPage;
+    constexpr int kTilesPerGroup = 32 / kPages;
     constexpr int kKBoxes = kPages * kHalves;  // K boxes per tile; V: kPages
     // lane -> its box: K (page, half) for lanes < kKBoxes, V page for the next kPages
     const int kb = lane < kKBoxes ? lane : 0;
@@ -179,11 +196,11 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
     int issued = 0;
     for (int j = 0; j < ntiles; ++j) {
       const int st = j % S;
-      if ((j & 7) == 0 && j > 0) {
+      if (j % kTilesPerGroup == 0 && j > 0) {
         cur = nxt;
-        nxt = fetch((j >> 3) + 1);
+        nxt = fetch(j / kTilesPerGroup + 1);
       }
-      const int bk = __shfl_sync(0xffffffffu, cur, (j & 7) * kPages + my_pg);
+      const int bk = __shfl_sync(0xffffffffu, cur, (j % kTilesPerGroup) * kPages + my_pg);
       const uint32_t ph = ((j / S) - 1) & 1;
       const uint32_t koff = st * L::kTileBytes + my_hf * (kTcTile * 128) + my_pg * (kPage * 128);
       const uint32_t voff = st * L::kTileBytes + my_pg * L::kPageBytes;
@@ -205,7 +222,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
         // the appended rows of this tile, straight from the input, over what
         // the pages held (generic writes, then a proxy fence for the MMA)
         const int key0 = kv_begin + j * kTcTile;
-        const int lo = max(key0, U.ctx), hi = min(key0 + kTcTile, U.kv_len);
+        const int lo = max(key0, U.ctx), hi = min(key0 + kTcTile, kv_end);
         const int n16 = (hi - lo) * (D / 8);
         go = true;
         if (lane == 0) go = mbar_wait(&k_full[st], (j / S) & 1, p.status);
@@ -263,12 +280,13 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
     // ----------------------------------------------------- MMA issuer (1 thread)
     if (lane == 0) {
       constexpr uint32_t kIdQK = idesc_bf16_f32(128, kTcTile, false, false);
-      constexpr uint32_t kIdPV = idesc_bf16_f32(128, 64, false, true);
+      constexpr uint32_t kIdPV = idesc_bf16_f32(128, D, false, true);
       const uint32_t k_addr = smem_addr(sK);
       const uint32_t v_addr = smem_addr(sV);
       bool ok = mbar_wait(q_ready, 0, p.status);
       int jq = 0, jp = 0;  // next Q K^T, next P V
       uint64_t idle_since = 0;
+      uint32_t idle_polls = 0;
       while (ok && jp < ntiles) {
         bool did = false;
         // S[jq & 1] is free once P V of tile jq - 2 has been issued (the
@@ -291,23 +309,25 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
             (patched(jp) ? mbar_test_wait(&v_patch[jp % S], 0) : mbar_test_wait(&v_full[jp % S], (jp / S) & 1))) {
           tc_fence_after();
           const uint32_t vt = v_addr + (jp % S) * L::kTileBytes;
-          const uint32_t pt = tS0 + (jp & 1) * kTcTile;  // P: 32 columns of bf16 pairs
+          const uint32_t pt = tS0 + (jp & 1) * kTcTile;  // P: 64 columns of bf16 pairs
 #pragma unroll
-          for (int hf = 0; hf < kHalves; ++hf) {
-#pragma unroll
-            for (int kk = 0; kk < kTcTile / 16; ++kk) {
-              const uint64_t bd = smem_desc_sw128(vt + kk * L::kPageBytes + hf * (kPage * 128), 1024, 1024);
-              tc_mma_ts(tO + hf * 64, pt + kk * 8, bd, kIdPV, (jp > 0 || kk > 0) ? 1u : 0u);
-            }
+          for (int kk = 0; kk < kTcTile / kPage; ++kk) {
+            // MN-major V page: 64-column halves kPage * 128 bytes apart
+            // (leading offset), 8-key groups 1024 bytes apart (stride offset)
+            const uint64_t bd = smem_desc_sw128(vt + kk * L::kPageBytes, kPage * 128, 1024);
+            tc_mma_ts(tO, pt + kk * 8, bd, kIdPV, (jp > 0 || kk > 0) ? 1u : 0u);
           }
           tc_commit(&pv_done[jp & 1]);
           tc_commit(&v_empty[jp % S]);
           ++jp;
           did = true;
         }
+        // the wait stays bounded, but the timer is read once per 256 idle
+        // polls: a %globaltimer read costs far more than a test_wait
         if (did) {
+          idle_polls = 0;
           idle_since = 0;
-        } else {
+        } else if ((++idle_polls & 255u) == 0) {
           const uint64_t now = global_timer_ns();
           if (idle_since == 0) {
             idle_since = now;
@@ -352,7 +372,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
       if (lane == 0) mbar_arrive(q_ready);
     }
 
-    const int last_vis = U.ctx + t;  // last visible key of this row
+    const int last_vis = min(U.ctx + t, kv_end - 1);  // last key of this row in this split
     // warps whose 32 rows are all padding write zero P, so every lane of P
     // the tensor core reads is defined
     const bool active = row0 + quad * 32 < M;
@@ -365,20 +385,17 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
       ok = __all_sync(0xffffffffu, mbar_wait(&s_full[b], (j >> 1) & 1, p.status));
       if (!ok) break;
       tc_fence_after();
-      uint32_t pk[kTcTile / 2];
-#pragma unroll
-      for (int c = 0; c < kTcTile / 2; ++c) pk[c] = 0u;
+      const uint32_t tSb = tS0 + b * kTcTile + lane_base;
       if (active) {
-        uint32_t sr[2][32];
-        tmem_ld32(tS0 + b * kTcTile + lane_base, sr[0]);
-        tmem_ld32(tS0 + b * kTcTile + 32 + lane_base, sr[1]);
+        uint32_t sr[kTcTile];
+        tmem_ld128(tSb, sr);
         // raw scores; the causal rule key <= C_i + t only bites near the end
         float s[kTcTile];
         float mr = -INFINITY;
-        const bool need_mask = key0 + kTcTile - 1 > U.ctx;
+        const bool need_mask = key0 + kTcTile - 1 > last_vis;
 #pragma unroll
         for (int c = 0; c < kTcTile; ++c) {
-          float v = __uint_as_float(sr[c >> 5][c & 31]);
+          float v = __uint_as_float(sr[c]);
           if (need_mask && key0 + c > last_vis) v = -INFINITY;
           s[c] = v;
           mr = fmaxf(mr, v);
@@ -407,17 +424,27 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
         }
         l *= factor;
         const float nb = m == -INFINITY ? 0.f : -m;
+        // P over the first 64 columns of S[b] (already read); the P V that
+        // read this buffer two tiles ago completed before S[b] was written
 #pragma unroll
-        for (int c = 0; c < kTcTile; c += 2) {
-          const float p0 = fast_exp2(__fmaf_rn(s[c], sl2, nb));
-          const float p1 = fast_exp2(__fmaf_rn(s[c + 1], sl2, nb));
-          l += p0 + p1;
-          pk[c >> 1] = pack_bf16x2(p0, p1);
+        for (int hh = 0; hh < kTcTile / 64; ++hh) {
+          uint32_t pk[32];
+#pragma unroll
+          for (int c = 0; c < 64; c += 2) {
+            const float p0 = fast_exp2(__fmaf_rn(s[hh * 64 + c], sl2, nb));
+            const float p1 = fast_exp2(__fmaf_rn(s[hh * 64 + c + 1], sl2, nb));
+            l += p0 + p1;
+            pk[c >> 1] = pack_bf16x2(p0, p1);
+          }
+          tmem_st32(tSb + hh * 32, pk);
         }
+      } else {
+        uint32_t pk[32];
+#pragma unroll
+        for (int c = 0; c < 32; ++c) pk[c] = 0u;
+#pragma unroll
+        for (int hh = 0; hh < kTcTile / 64; ++hh) tmem_st32(tSb + hh * 32, pk);
       }
-      // P over the first 32 columns of S[b] (already read); the P V that
-      // read this buffer two tiles ago completed before S[b] was written
-      tmem_st32(tS0 + b * kTcTile + lane_base, pk);
       // V rows past kv_len may hold anything; zero them before P V reads them
       if (key0 + kTcTile > U.kv_len) {
         ok = __all_sync(0xffffffffu, mbar_wait(&v_full[st], (j / S) & 1, p.status));
@@ -476,7 +503,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
 
   if (p.cluster > 1) {
     // ---- split merge inside the cluster (every thread takes both barriers)
-    constexpr int kSlot = 128 * 8 + 128 * D * 4;  // (m, l) per row, then O as [D/4][128] float4
+    constexpr int kSlot = L::kSlotBytes;  // (m, l) per row, then O as [D/4][128] float4
     const uint32_t crank = cluster_ctarank();
     const int quad = warp & 3;
     const int r = quad * 32 + lane;

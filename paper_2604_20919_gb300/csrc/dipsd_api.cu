@@ -166,17 +166,22 @@ int check_attn_users(int B, const int* L, const int* ctx, int Hq, int Hkv, int D
   return DIPSD_OK;
 }
 
-// Chooses the KV split length (a multiple of the 64-token tile) that
-// minimises a list-scheduling estimate of the makespan over the resident CTA
-// slots: total work / slots + the largest item, with a per-item overhead of
-// two tiles (prologue, pipeline fill, epilogue) and the merge traffic.
+// Chooses how many KV splits each user gets, minimising a list-scheduling
+// estimate of the makespan over the resident CTA slots: total work / slots +
+// the largest item, with a per-item overhead (prologue, pipeline fill,
+// epilogue) and the merge traffic.  A user's splits are as even as whole
+// 16-token pages allow (the kernel masks a split's last tile at its end).
+// Costs are in units of 64 tokens of one (user, head) stream.
+// Pages per split when `pages` pages are cut into `ns` near-equal splits.
+static int split_pages(int pages, int ns) { return (pages + ns - 1) / ns; }
+
 void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int Hq, int Hkv, int D,
                     int sms, AttnPlan& pl) {
   pl.B = B; pl.Hq = Hq; pl.Hkv = Hkv; pl.G = Hq / Hkv; pl.D = D;
   int max_m = 0, max_tiles = 1;
   for (int i = 0; i < B; ++i) {
     max_m = std::max(max_m, pl.G * (L[i] + 1));
-    max_tiles = std::max(max_tiles, (ctx[i] + L[i] + 1 + kAttnTile - 1) / kAttnTile);
+    max_tiles = std::max(max_tiles, (ctx[i] + L[i] + 1 + kTcTile - 1) / kTcTile);
   }
   // tcgen05 kernel: 128 rows per CTA, one CTA per SM (its shared memory)
   pl.NW = 8;
@@ -200,13 +205,14 @@ void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int
     long long items = 0;
     bool any_split = false;
     for (int i = 0; i < B; ++i) {
-      const int tiles = (ctx[i] + L[i] + 1 + kAttnTile - 1) / kAttnTile;
+      const int tiles = (ctx[i] + L[i] + 1 + kTcTile - 1) / kTcTile;
+      const int pages = (ctx[i] + L[i] + 1 + kPage - 1) / kPage;
       const int cc = std::max(1, std::min(c, tiles));
       int ns = (tiles + cc - 1) / cc;
-      const int st = (tiles + ns - 1) / ns;
-      ns = (tiles + st - 1) / st;
+      const int sp = split_pages(pages, ns);
+      ns = (pages + sp - 1) / sp;
       const int rb = (pl.G * (L[i] + 1) + rows_cta - 1) / rows_cta;
-      const double item = st + 2.0 + (ns > 1 ? 0.5 : 0.0);
+      const double item = sp * kPage / 64.0 + 2.0 + (ns > 1 ? 0.5 : 0.0);
       total += item * ns * rb * Hkv;
       items += static_cast<long long>(ns) * rb * Hkv;
       max_item = std::max(max_item, item);
@@ -223,7 +229,7 @@ void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int
 
   // Cluster merge: every user's KV in the same number C of splits (one wave,
   // the exchange buffer of C - 1 ranks fitting rank 0's rings).
-  const int max_cluster = D == 128 ? 3 : 6;
+  const int max_cluster = D == 128 ? TcSmem<128>::kMaxCluster : TcSmem<64>::kMaxCluster;
   int best_cl = 0;
   double best_b = 1e300;
   for (int C = 2; C <= max_cluster && forced == 0; ++C) {
@@ -231,10 +237,10 @@ void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int
     long long items = 0;
     double max_item = 0;
     for (int i = 0; i < B; ++i) {
-      const int tiles = (ctx[i] + L[i] + 1 + kAttnTile - 1) / kAttnTile;
+      const int pages = (ctx[i] + L[i] + 1 + kPage - 1) / kPage;
       const int rb = (pl.G * (L[i] + 1) + rows_cta - 1) / rows_cta;
       items += static_cast<long long>(C) * rb * Hkv;
-      max_item = std::max(max_item, (tiles + C - 1) / C + 2.5);
+      max_item = std::max(max_item, split_pages(pages, C) * kPage / 64.0 + 2.5);
     }
     if (items <= slots || forced_cluster > 0) {
       if (max_item < best_b) { best_b = max_item; best_cl = C; }
@@ -255,19 +261,20 @@ void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int
     U.T = L[i] + 1;
     U.kv_len = ctx[i] + U.T;
     U.bt_row = bt_rows ? bt_rows[i] : i;
-    const int tiles = (U.kv_len + kAttnTile - 1) / kAttnTile;
-    int ns, st;
+    const int tiles = (U.kv_len + kTcTile - 1) / kTcTile;
+    const int pages = (U.kv_len + kPage - 1) / kPage;
+    int ns, sp;
     if (pl.cluster > 1) {
-      ns = pl.cluster;  // trailing splits may be empty when tiles < C
-      st = (tiles + ns - 1) / ns;
+      ns = pl.cluster;  // trailing splits may be empty when pages < C
+      sp = split_pages(pages, ns);
     } else {
       const int cc = std::max(1, std::min(best_c, tiles));
       ns = (tiles + cc - 1) / cc;
-      st = (tiles + ns - 1) / ns;
-      ns = (tiles + st - 1) / st;
+      sp = split_pages(pages, ns);
+      ns = (pages + sp - 1) / sp;
     }
     U.nsplit = ns;
-    U.split_len = st * kAttnTile;
+    U.split_len = sp * kPage;
     U.n_rb = (pl.G * U.T + rows_cta - 1) / rows_cta;
     pl.item_off[i] = static_cast<int>(items);
     pl.merge_off[i] = static_cast<int>(merge);

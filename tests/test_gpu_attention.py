@@ -48,6 +48,7 @@ def test_attention_long_context_sampled_users(cuda_lib):
 @pytest.mark.parametrize("L,ctx,Hq,Hkv,D", [
     ([0, 0, 0], [0, 1, 15], 8, 2, 128),          # kv_len 1, 2, 16: single page, tiny
     ([3, 0, 7, 1], [16, 47, 63, 64], 64, 8, 128),  # page and tile edges
+    ([0, 2, 5, 0], [127, 126, 250, 383], 64, 8, 128),  # kv_len 128, 129, 256, 384: 128-key tile edges
     ([31, 16], [5, 200], 64, 8, 128),            # G*T = 256 and 136: two row blocks
     ([9, 2], [300, 1000], 64, 8, 128),           # G*T = 80: eight consumer warps
     ([4, 1, 2], [129, 1, 700], 4, 1, 64),        # head_dim 64, G = 4
