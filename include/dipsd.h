@@ -184,7 +184,11 @@ int dipsd_spec_verify_sparse(int B, const int* h_L, int V, int K, int logit_dtyp
 
 /* ------------------------------------------------------------------------
  * One pipeline stage: the users of batch n (Sec. III-C, B_n(x)) verified
- * together -- attention, then speculative verification, on one stream.
+ * together -- attention and speculative verification, on one stream.  The
+ * two stages read disjoint inputs and run overlapped (the attention grid
+ * streams the KV cache while the sampling kernel finishes); all outputs are
+ * complete when the work queued on the stream completes.  No output buffer
+ * may overlap an input buffer.
  *
  * Per-user tables cover all M users being served; h_members[b] (distinct, in
  * [0, M)) names the b-th user of this batch.  Per-batch tensors (d_q,

@@ -41,6 +41,11 @@ struct AttnParams {
   __nv_bfloat16* k_cache;  // [num_blocks][Hkv][16][D], written only when new_k is set
   __nv_bfloat16* v_cache;
   int num_blocks;          // cache blocks (bound for the append writes)
+  // 1: the kernel reads nothing the preceding grid writes (it runs after the
+  // spec_verify kernels of the same batch, whose own wait covered everything
+  // before the call), so it waits for that grid only before it exits: the
+  // launch then completes only after both stages have
+  int wait_at_end;
   int cluster;  // > 1: the nsplit == cluster splits of a row block and head
                 // form one thread-block cluster and merge in shared memory
   int B, Hq, Hkv, G, max_blocks;

@@ -169,7 +169,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
   const uint32_t tS0 = tmem, tO = tmem + 2 * kTcTile, tQ = tmem + 384;
   float fin_m = -INFINITY, fin_l = 0.f;  // softmax threads: row state after the last tile
   bool fin_ok = false;
-  pdl_wait_prior_grid();
+  if (!p.wait_at_end) pdl_wait_prior_grid();
   pdl_launch_dependents();
 
   if (warp == 0) {
@@ -590,6 +590,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
+  if (p.wait_at_end && threadIdx.x == 0) pdl_wait_prior_grid();
 }
 
 }  // namespace dipsd

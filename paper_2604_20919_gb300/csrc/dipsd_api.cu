@@ -341,9 +341,10 @@ int launch_attention_tc_t(const AttnPlan& pl, const AttnParams<CAP>& p, const CU
 template <int CAP>
 int run_attention_cap(const AttnPlan& pl, const void* q, const void* kc, const void* vc, int num_blocks,
                       const int* bt, int max_blocks, float scale, void* out, unsigned* status,
-                      uint8_t* region, cudaStream_t s, bool pdl, const KvAppend& app) {
+                      uint8_t* region, cudaStream_t s, bool pdl, const KvAppend& app, bool wait_at_end) {
   static thread_local AttnParams<CAP> p;
   fill_attn_params<CAP>(p, pl, q, out, bt, max_blocks, scale, status, region);
+  p.wait_at_end = wait_at_end ? 1 : 0;
   p.new_k = static_cast<const __nv_bfloat16*>(app.new_k);
   p.new_v = static_cast<const __nv_bfloat16*>(app.new_v);
   p.k_cache = static_cast<__nv_bfloat16*>(const_cast<void*>(kc));
@@ -359,12 +360,12 @@ int run_attention_cap(const AttnPlan& pl, const void* q, const void* kc, const v
 
 int run_attention(const AttnPlan& pl, const void* q, const void* kc, const void* vc, int num_blocks,
                   const int* bt, int max_blocks, float scale, void* out, unsigned* status, uint8_t* region,
-                  cudaStream_t s, bool pdl, const KvAppend& app = KvAppend{}) {
+                  cudaStream_t s, bool pdl, const KvAppend& app = KvAppend{}, bool wait_at_end = false) {
   if (pl.B <= kCapSmall)
     return run_attention_cap<kCapSmall>(pl, q, kc, vc, num_blocks, bt, max_blocks, scale, out, status,
-                                        region, s, pdl, app);
+                                        region, s, pdl, app, wait_at_end);
   return run_attention_cap<kCapLarge>(pl, q, kc, vc, num_blocks, bt, max_blocks, scale, out, status,
-                                      region, s, pdl, app);
+                                      region, s, pdl, app, wait_at_end);
 }
 
 int check_append(const void* new_k, const void* new_v, const void* q) {
@@ -896,11 +897,16 @@ static int verify_batch_impl(int B, const int* h_members, int M, const int* h_L_
   uint8_t* ws = static_cast<uint8_t*>(d_workspace);
   unsigned* status = reinterpret_cast<unsigned*>(ws);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  st = run_attention(ap, d_q, d_k_cache, d_v_cache, num_blocks, d_block_table_all, max_blocks, softmax_scale,
-                     d_attn_out, status, ws + kHeaderBytes, s, true, app);
-  if (st != DIPSD_OK) return st;
+  // The two stages share no data.  spec_verify goes first; the attention
+  // grid launches as soon as the sampling kernel has passed its own wait
+  // (so everything before this call is complete), streams the KV cache
+  // while the sampling kernel's per-user descents finish, and waits for
+  // that kernel only before it exits.
   st = run_spec(sp, logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
                 d_out_offsets, d_out_tokens, d_draft_probs, status, ws + kHeaderBytes + attn_region, s, true);
+  if (st != DIPSD_OK) return st;
+  st = run_attention(ap, d_q, d_k_cache, d_v_cache, num_blocks, d_block_table_all, max_blocks, softmax_scale,
+                     d_attn_out, status, ws + kHeaderBytes, s, true, app, true);
   return st != DIPSD_OK ? st : cuda_status();
 }
 
