@@ -15,9 +15,8 @@
 //               128 bytes), stored page after page.  K and V stages are
 //               released separately: K once its Q K^T has run, V after its
 //               P V.  Page ids are fetched 32 at a time, one per lane, a
-//               group ahead; pages past the user's end are requested at an
-//               out-of-range block, which TMA fills with zeros without
-//               reading memory.
+//               group ahead.  A split's last tile loads only the pages up
+//               to the split's end.
 //   warp 1      allocates TMEM; one thread issues tcgen05.mma as operands
 //               become ready (no fixed order between the two products):
 //                 S[b] = Q K^T      (A = Q from tensor memory, M=128, N=128)
@@ -42,9 +41,10 @@
 // pages (the round's state update).
 // KV splits: either each split writes (m, l, O) rows to global memory for
 // verify_attention_merge_kernel, or (p.cluster > 1) the splits of one row
-// block and head run as one thread-block cluster: the other ranks push their
-// rows into rank 0's drained rings through distributed shared memory and
-// rank 0 merges them with its own O straight from TMEM.
+// block and head run as one thread-block cluster and merge through
+// distributed shared memory: each rank owns a share of the 32-column chunks
+// of O, receives the other ranks' (m, l) rows and their rows of its chunks in
+// its drained K ring, and writes those columns of the output.
 // TMEM columns: S/P double buffer [0,128) [128,256), O [256, 256+D), Q
 // [384, 384 + D/2).  Shared memory holds only the two rings (Q and P live in
 // tensor memory, so no product re-reads an operand from shared memory every
@@ -72,13 +72,16 @@ struct TcSmem {
   static constexpr int kBarOff = kVOff + kStages * kTileBytes;
   static constexpr int kBytes = kBarOff + 1024;  // barriers (6 kStages + 8) and the TMEM slot
   static constexpr int kAlloc = kBytes + 1024;  // slack for 1024-byte alignment
-  // cluster merge: the other ranks' (m, l, O) rows land in rank 0's drained
-  // rings, up to kMaxCluster - 1 of them
+  // cluster merge: rank r finalises the 32-column chunks cc with cc % C == r;
+  // every other rank's (m, l) rows and its O rows of those chunks land in one
+  // slot of r's drained K ring, up to kMaxCluster - 1 slots
+  static constexpr int kChunks = D / 32;
   static constexpr int kMaxCluster = D == 128 ? 3 : 6;
-  static constexpr int kSlotBytes = 128 * 8 + 128 * D * 4;
+  static constexpr int kChunkBytes = 128 * 32 * 4;
+  static constexpr int kSlotBytes = 128 * 8 + ((kChunks + 1) / 2) * kChunkBytes;
 };
-static_assert((TcSmem<128>::kMaxCluster - 1) * TcSmem<128>::kSlotBytes <= TcSmem<128>::kBarOff, "exchange fits");
-static_assert((TcSmem<64>::kMaxCluster - 1) * TcSmem<64>::kSlotBytes <= TcSmem<64>::kBarOff, "exchange fits");
+static_assert((TcSmem<128>::kMaxCluster - 1) * TcSmem<128>::kSlotBytes <= TcSmem<128>::kVOff, "exchange fits");
+static_assert((TcSmem<64>::kMaxCluster - 1) * TcSmem<64>::kSlotBytes <= TcSmem<64>::kVOff, "exchange fits");
 static_assert(TcSmem<128>::kAlloc <= 232448 && TcSmem<64>::kAlloc <= 232448, "shared memory per CTA");
 constexpr int kTcStages = TcSmem<128>::kStages;
 
@@ -124,8 +127,11 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
   const int kv_begin = split * U.split_len;
   const int kv_end = min(kv_begin + U.split_len, U.kv_len);
   const int ntiles = max(0, (kv_end - kv_begin + kTcTile - 1) / kTcTile);  // 0: an empty split
-  // Splits start on a page; a split's last tile may run past kv_end into the
-  // next split's keys, which are masked and never loaded.
+  // Splits start on a page.  A split's last tile holds only the pages up to
+  // kv_end: only those are loaded, multiplied (Q K^T with N = 16 per page,
+  // one P V step per page) and run through the softmax.
+  const int split_pages_n = (kv_end + kPage - 1) / kPage - kv_begin / kPage;
+  auto tile_pages = [&](int j) { return min(kTcTile / kPage, split_pages_n - j * (kTcTile / kPage)); };
   // tile j holds new (appended) rows: keys [max(key0, C_i), min(key0 + 128, kv_end))
   auto patched = [&](int j) {
     const int key0 = kv_begin + j * kTcTile;
@@ -181,7 +187,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
     const int page_base = kv_begin / kPage;
     auto fetch = [&](int group) {
       const int page = page_base + group * 32 + lane;
-      return page < n_pages ? __ldg(bt + page) : p.num_blocks;  // past the end: zero fill
+      return page < n_pages ? __ldg(bt + page) : p.num_blocks;  // past the end: never requested
     };
     constexpr int kPages = kTcTile / kPage;
     constexpr int kTilesPerGroup = 32 / kPages;
@@ -204,19 +210,21 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
       const uint32_t ph = ((j / S) - 1) & 1;
       const uint32_t koff = st * L::kTileBytes + my_hf * (kTcTile * 128) + my_pg * (kPage * 128);
       const uint32_t voff = st * L::kTileBytes + my_pg * L::kPageBytes;
+      const int tp = tile_pages(j);  // pages of this tile (kPages except in a split's last tile)
       // K tile
       bool go = true;
       if (j >= S && lane == 0) go = mbar_wait(&k_empty[st], ph, p.status);
       if (!__shfl_sync(0xffffffffu, go, 0)) break;
-      if (lane == 0) mbar_arrive_expect_tx(&k_full[st], L::kTileBytes);
+      if (lane == 0) mbar_arrive_expect_tx(&k_full[st], tp * L::kPageBytes);
       __syncwarp();
-      if (lane < kKBoxes) tma_load_4d(sK + koff, &tm_k, my_hf * 64, 0, h, bk, &k_full[st]);
+      if (lane < kKBoxes && my_pg < tp) tma_load_4d(sK + koff, &tm_k, my_hf * 64, 0, h, bk, &k_full[st]);
       // V tile
       if (j >= S && lane == 0) go = mbar_wait(&v_empty[st], ph, p.status);
       if (!__shfl_sync(0xffffffffu, go, 0)) break;
-      if (lane == 0) mbar_arrive_expect_tx(&v_full[st], L::kTileBytes);
+      if (lane == 0) mbar_arrive_expect_tx(&v_full[st], tp * L::kPageBytes);
       __syncwarp();
-      if (lane >= kKBoxes && lane < kKBoxes + kPages) tma_load_5d(sV + voff, &tm_v, 0, 0, 0, h, bk, &v_full[st]);
+      if (lane >= kKBoxes && lane < kKBoxes + kPages && my_pg < tp)
+        tma_load_5d(sV + voff, &tm_v, 0, 0, 0, h, bk, &v_full[st]);
       ++issued;
       if (patched(j)) {
         // the appended rows of this tile, straight from the input, over what
@@ -295,10 +303,12 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
             (patched(jq) ? mbar_test_wait(&k_patch[jq % S], 0) : mbar_test_wait(&k_full[jq % S], (jq / S) & 1))) {
           tc_fence_after();
           const uint32_t kt = k_addr + (jq % S) * L::kTileBytes;
+          // N = 16 keys per loaded page
+          const uint32_t id_qk = jq + 1 < ntiles ? kIdQK : idesc_bf16_f32(128, tile_pages(jq) * kPage, false, false);
 #pragma unroll
           for (int kk = 0; kk < D / 16; ++kk) {
             const uint64_t bd = smem_desc_sw128(kt + (kk >> 2) * (kTcTile * 128) + (kk & 3) * 32, 0, 1024);
-            tc_mma_ts(tS0 + (jq & 1) * kTcTile, tQ + kk * 8, bd, kIdQK, kk > 0 ? 1u : 0u);
+            tc_mma_ts(tS0 + (jq & 1) * kTcTile, tQ + kk * 8, bd, id_qk, kk > 0 ? 1u : 0u);
           }
           tc_commit(&s_full[jq & 1]);
           tc_commit(&k_empty[jq % S]);
@@ -310,8 +320,10 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
           tc_fence_after();
           const uint32_t vt = v_addr + (jp % S) * L::kTileBytes;
           const uint32_t pt = tS0 + (jp & 1) * kTcTile;  // P: 64 columns of bf16 pairs
+          const int np = tile_pages(jp);
 #pragma unroll
           for (int kk = 0; kk < kTcTile / kPage; ++kk) {
+            if (kk >= np) break;
             // MN-major V page: 64-column halves kPage * 128 bytes apart
             // (leading offset), 8-key groups 1024 bytes apart (stride offset)
             const uint64_t bd = smem_desc_sw128(vt + kk * L::kPageBytes, kPage * 128, 1024);
@@ -386,15 +398,20 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
       if (!ok) break;
       tc_fence_after();
       const uint32_t tSb = tS0 + b * kTcTile + lane_base;
-      if (active) {
-        uint32_t sr[kTcTile];
-        tmem_ld128(tSb, sr);
+      // one tile's softmax over its first NC score columns (NC = 128, or 32
+      // for a last tile of at most two pages); false: a wait gave up
+      auto tile_softmax = [&](auto nc_tag) -> bool {
+        constexpr int NC = decltype(nc_tag)::value;
+        uint32_t sr[NC];
+        if constexpr (NC == 128) tmem_ld128(tSb, sr);
+        else tmem_ld32(tSb, sr);
         // raw scores; the causal rule key <= C_i + t only bites near the end
-        float s[kTcTile];
+        // (columns past the tile's pages are keys past kv_end: masked too)
+        float s[NC];
         float mr = -INFINITY;
-        const bool need_mask = key0 + kTcTile - 1 > last_vis;
+        const bool need_mask = key0 + NC - 1 > last_vis;
 #pragma unroll
-        for (int c = 0; c < kTcTile; ++c) {
+        for (int c = 0; c < NC; ++c) {
           float v = __uint_as_float(sr[c]);
           if (need_mask && key0 + c > last_vis) v = -INFINITY;
           s[c] = v;
@@ -410,8 +427,8 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
         }
         if (j > 0 && __any_sync(0xffffffffu, grow && factor != 1.f)) {
           // every earlier P V has to be done before O is touched
-          ok = __all_sync(0xffffffffu, mbar_wait(&pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1, p.status));
-          if (!ok) break;
+          if (!__all_sync(0xffffffffu, mbar_wait(&pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1, p.status)))
+            return false;
           tc_fence_after();
 #pragma unroll
           for (int cc = 0; cc < D / 32; ++cc) {
@@ -424,20 +441,29 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
         }
         l *= factor;
         const float nb = m == -INFINITY ? 0.f : -m;
-        // P over the first 64 columns of S[b] (already read); the P V that
+        // P over the first NC / 2 columns of S[b] (already read); the P V that
         // read this buffer two tiles ago completed before S[b] was written
+        constexpr int kPk = NC < 64 ? NC / 2 : 32;
 #pragma unroll
-        for (int hh = 0; hh < kTcTile / 64; ++hh) {
-          uint32_t pk[32];
+        for (int hh = 0; hh < (NC + 63) / 64; ++hh) {
+          uint32_t pk[kPk];
 #pragma unroll
-          for (int c = 0; c < 64; c += 2) {
+          for (int c = 0; c < 2 * kPk; c += 2) {
             const float p0 = fast_exp2(__fmaf_rn(s[hh * 64 + c], sl2, nb));
             const float p1 = fast_exp2(__fmaf_rn(s[hh * 64 + c + 1], sl2, nb));
             l += p0 + p1;
             pk[c >> 1] = pack_bf16x2(p0, p1);
           }
-          tmem_st32(tSb + hh * 32, pk);
+          if constexpr (kPk == 32) tmem_st32(tSb + hh * 32, pk);
+          else tmem_st16(tSb + hh * 32, pk);
         }
+        return true;
+      };
+      if (active) {
+        const bool done = tile_pages(j) * kPage <= 32 ? tile_softmax(std::integral_constant<int, 32>{})
+                                                      : tile_softmax(std::integral_constant<int, kTcTile>{});
+        ok = done;
+        if (!ok) break;
       } else {
         uint32_t pk[32];
 #pragma unroll
@@ -450,8 +476,8 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
         ok = __all_sync(0xffffffffu, mbar_wait(&v_full[st], (j / S) & 1, p.status));
         if (!ok) break;
         uint8_t* vt = sV + st * L::kTileBytes;
-        const int first = U.kv_len - key0;  // first key row to clear
-        const int nchunks = (kTcTile - first) * kHalves * 8;
+        const int first = U.kv_len - key0;  // first key row to clear, up to the tile's loaded pages
+        const int nchunks = max(0, tile_pages(j) * kPage - first) * kHalves * 8;
         for (int c = threadIdx.x - 64; c < nchunks; c += 128) {
           const int row = first + c / (kHalves * 8);
           const int rem = c % (kHalves * 8);  // every 16-byte chunk of the row, in any order
@@ -502,68 +528,80 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
   }
 
   if (p.cluster > 1) {
-    // ---- split merge inside the cluster (every thread takes both barriers)
-    constexpr int kSlot = L::kSlotBytes;  // (m, l) per row, then O as [D/4][128] float4
-    const uint32_t crank = cluster_ctarank();
+    // ---- split merge inside the cluster (every thread takes both barriers).
+    // Rank r finalises the 32-column chunks cc with cc % C == r.  Every rank
+    // pushes its (m, l) rows to all others and each chunk it does not own to
+    // the owner; the owner weighs the C partial rows by 2^(m_s - max m) and
+    // writes its columns of the output.
+    constexpr int kSlot = L::kSlotBytes;  // (m, l) per row, then the owner's chunks as [8][128] float4
+    constexpr int kCh = L::kChunks;
+    const int C = p.cluster;
+    const int crank = static_cast<int>(cluster_ctarank());
     const int quad = warp & 3;
     const int r = quad * 32 + lane;
     const int rg = row0 + r;
     const bool valid = rg < M;
     const bool active = warp >= 2 && row0 + quad * 32 < M;
     const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;
-    uint8_t* xbuf = sK;  // rank 0's rings, drained once every rank is here
+    uint8_t* xbuf = sK;  // every rank's K ring, drained once all ranks are here
+    // slot of source rank `src` at receiving rank `dst`
+    auto slot_of = [&](int src, int dst) { return (src < dst ? src : src - 1) * kSlot; };
     cluster_arrive_release();
     cluster_wait_acquire();
-    if (active && crank > 0 && fin_ok) {
-      const uint32_t slot = dsmem_map(xbuf + (crank - 1) * kSlot, 0);
-      if (valid) dsmem_st_f32x2(slot + r * 8, fin_m, fin_l);
+    if (active && fin_ok) {
+      for (int dst = 0; dst < C; ++dst)
+        if (dst != crank && valid) dsmem_st_f32x2(dsmem_map(xbuf + slot_of(crank, dst), dst) + r * 8, fin_m, fin_l);
       tc_fence_after();
 #pragma unroll 1
-      for (int cc = 0; cc < D / 32; ++cc) {
+      for (int cc = 0; cc < kCh; ++cc) {
+        const int dst = cc % C;
+        if (dst == crank) continue;
         uint32_t o[32];
         tmem_ld32(tO + cc * 32 + lane_base, o);
         if (valid && fin_l > 0.f) {
+          const uint32_t base = dsmem_map(xbuf + slot_of(crank, dst), dst) + 1024 + (cc / C) * L::kChunkBytes;
 #pragma unroll
           for (int k = 0; k < 8; ++k)
-            dsmem_st_f32x4(slot + 1024 + ((cc * 8 + k) * 128 + r) * 16, __uint_as_float(o[4 * k]),
-                           __uint_as_float(o[4 * k + 1]), __uint_as_float(o[4 * k + 2]),
-                           __uint_as_float(o[4 * k + 3]));
+            dsmem_st_f32x4(base + (k * 128 + r) * 16, __uint_as_float(o[4 * k]), __uint_as_float(o[4 * k + 1]),
+                           __uint_as_float(o[4 * k + 2]), __uint_as_float(o[4 * k + 3]));
         }
       }
     }
     cluster_arrive_release();
     cluster_wait_acquire();
-    if (active && crank == 0 && fin_ok) {
-      const int C = p.cluster;
+    if (active && fin_ok && crank < kCh) {
       const int t = rg / p.G, g = rg % p.G;
       float mx = fin_m;
-      for (int s = 1; s < C; ++s)
-        mx = fmaxf(mx, reinterpret_cast<const float2*>(xbuf + (s - 1) * kSlot)[r].x);
+      for (int s = 0; s < C; ++s)
+        if (s != crank) mx = fmaxf(mx, reinterpret_cast<const float2*>(xbuf + slot_of(s, crank))[r].x);
       // weights 2^(m_s - mx) (log2 units); an empty split weighs 0
       const float w0 = fin_m == -INFINITY ? 0.f : fast_exp2(fin_m - mx);
       float l = w0 * fin_l;
-      for (int s = 1; s < C; ++s) {
-        const float2 ml = reinterpret_cast<const float2*>(xbuf + (s - 1) * kSlot)[r];
+      for (int s = 0; s < C; ++s) {
+        if (s == crank) continue;
+        const float2 ml = reinterpret_cast<const float2*>(xbuf + slot_of(s, crank))[r];
         l += ml.x == -INFINITY ? 0.f : fast_exp2(ml.x - mx) * ml.y;
       }
       const float inv = l > 0.f ? 1.f / l : 0.f;
       __nv_bfloat16* orow = p.out + (static_cast<size_t>(U.q_off + t) * p.Hq + h * p.G + g) * D;
       tc_fence_after();
 #pragma unroll 1
-      for (int cc = 0; cc < D / 32; ++cc) {
+      for (int cc = crank; cc < kCh; cc += C) {
         uint32_t o[32];
         tmem_ld32(tO + cc * 32 + lane_base, o);
         float acc[32];
 #pragma unroll
         for (int k = 0; k < 32; ++k) acc[k] = w0 > 0.f ? w0 * __uint_as_float(o[k]) : 0.f;
-        for (int s = 1; s < C; ++s) {
-          const float2 ml = reinterpret_cast<const float2*>(xbuf + (s - 1) * kSlot)[r];
+        for (int s = 0; s < C; ++s) {
+          if (s == crank) continue;
+          const float2 ml = reinterpret_cast<const float2*>(xbuf + slot_of(s, crank))[r];
           if (!(ml.x > -INFINITY) || !(ml.y > 0.f)) continue;
           const float w = fast_exp2(ml.x - mx);
-          const float4* os = reinterpret_cast<const float4*>(xbuf + (s - 1) * kSlot + 1024);
+          const float4* os =
+              reinterpret_cast<const float4*>(xbuf + slot_of(s, crank) + 1024 + (cc / C) * L::kChunkBytes);
 #pragma unroll
           for (int k = 0; k < 8; ++k) {
-            const float4 v = os[(cc * 8 + k) * 128 + r];
+            const float4 v = os[k * 128 + r];
             acc[4 * k] += w * v.x;
             acc[4 * k + 1] += w * v.y;
             acc[4 * k + 2] += w * v.z;
