@@ -492,37 +492,20 @@ __device__ __forceinline__ void vec_weights_table(const uint4& rz, const float (
 }
 
 // ----------------------------------------------------- position decision
-// Run by the warp that delivered the last segment of position q0 + t of user
-// ui: row sums, p_t(d), q_t(d), the acceptance decision; the user's last
-// decided position also writes a_i.
+// The decision of position q0 + t of user ui from the row sums (integer
+// reference, float-float sum) of z_t and w_t and the draft token's logits zd,
+// wd (NaN: the token lies outside [0, V)) or, for a sparse payload, log q(d):
+// SpecStat, p_t(d) and q_t(d), and the acceptance bit, added to the user's
+// decision word (arrivals in the high half); the user's last decided
+// position writes a_i.  One thread.
 template <int CAP, bool SP>
-__device__ __forceinline__ void decide_position(const SpecParams<CAP>& p, int ui, int t, int lane) {
+__device__ __forceinline__ void decide_from_sums(const SpecParams<CAP>& p, int ui, int t, RefSum az, RefSum aw,
+                                                 float zd, float wd, float logq) {
   const int q0 = p.q_off[ui];
   const int Li = p.q_off[ui + 1] - q0 - 1;
-  const int n = q0 + t, l = p.l_off[ui] + t;
+  const int n = q0 + t;
   const bool has_q = t < Li;
-  const float4* pz = p.part1 + static_cast<size_t>(n) * p.nseg1;
-  const float4* pw = p.part1 + static_cast<size_t>(p.sum_t + l) * p.nseg1;
-  // every load first: the draft token's logits, left by the rows' first
-  // segments (NaN: d outside [0, V)), and both rows' segment partials
-  float zd = 0.f, wd = 0.f, logq = 0.f;
-  if (has_q && lane == 0) {
-    zd = __ldcg(&pz->w);
-    if constexpr (SP) logq = p.draft_logq[l];
-    else wd = __ldcg(&pw->w);
-  }
-  RefSum az{kEmptyRef, FF{0.f, 0.f}}, aw{kEmptyRef, FF{0.f, 0.f}};
-#pragma unroll 2
-  for (int sg = lane; sg < p.nseg1; sg += 32) {
-    const float4 vz = __ldcg(pz + sg);
-    const float4 vw = has_q && !SP ? __ldcg(pw + sg) : make_float4(__int_as_float(kEmptyRef), 0.f, 0.f, 0.f);
-    az = refsum_add(az, RefSum{__float_as_int(vz.x), FF{vz.y, vz.z}});
-    aw = refsum_add(aw, RefSum{__float_as_int(vw.x), FF{vw.y, vw.z}});
-  }
-  az = warp_refsum(az);
-  if (has_q && !SP) aw = warp_refsum(aw);
-  if (lane == 0) {
-    p.counters[n] = 0u;
+  {
     SpecStat st;
     st.sz = static_cast<double>(az.s.hi) + static_cast<double>(az.s.lo);
     st.cz = az.c;
@@ -579,6 +562,41 @@ __device__ __forceinline__ void decide_position(const SpecParams<CAP>& p, int ui
       p.accept_len[ui] = min(__ffs(~static_cast<unsigned>(now)) - 1, Li);
       *word = 0ull;
     }
+  }
+}
+
+// Run by the warp that delivered the last segment of position q0 + t of user
+// ui: row sums, p_t(d), q_t(d), the acceptance decision; the user's last
+// decided position also writes a_i.
+template <int CAP, bool SP>
+__device__ __forceinline__ void decide_position(const SpecParams<CAP>& p, int ui, int t, int lane) {
+  const int q0 = p.q_off[ui];
+  const int Li = p.q_off[ui + 1] - q0 - 1;
+  const int n = q0 + t, l = p.l_off[ui] + t;
+  const bool has_q = t < Li;
+  const float4* pz = p.part1 + static_cast<size_t>(n) * p.nseg1;
+  const float4* pw = p.part1 + static_cast<size_t>(p.sum_t + l) * p.nseg1;
+  // every load first: the draft token's logits, left by the rows' first
+  // segments (NaN: d outside [0, V)), and both rows' segment partials
+  float zd = 0.f, wd = 0.f, logq = 0.f;
+  if (has_q && lane == 0) {
+    zd = __ldcg(&pz->w);
+    if constexpr (SP) logq = p.draft_logq[l];
+    else wd = __ldcg(&pw->w);
+  }
+  RefSum az{kEmptyRef, FF{0.f, 0.f}}, aw{kEmptyRef, FF{0.f, 0.f}};
+#pragma unroll 2
+  for (int sg = lane; sg < p.nseg1; sg += 32) {
+    const float4 vz = __ldcg(pz + sg);
+    const float4 vw = has_q && !SP ? __ldcg(pw + sg) : make_float4(__int_as_float(kEmptyRef), 0.f, 0.f, 0.f);
+    az = refsum_add(az, RefSum{__float_as_int(vz.x), FF{vz.y, vz.z}});
+    aw = refsum_add(aw, RefSum{__float_as_int(vw.x), FF{vw.y, vw.z}});
+  }
+  az = warp_refsum(az);
+  if (has_q && !SP) aw = warp_refsum(aw);
+  if (lane == 0) {
+    p.counters[n] = 0u;
+    decide_from_sums<CAP, SP>(p, ui, t, az, aw, zd, wd, logq);
   }
 }
 
@@ -646,17 +664,6 @@ __device__ __forceinline__ void descend(const SpecParams<CAP>& p, int ui, int a,
   constexpr int N = Vec16<T>::N;
   const int q0 = p.q_off[ui], l0 = p.l_off[ui];
   const int n = q0 + a;
-  if (lane == 0) p.counters[kCntUser2 + ui] = 0u;
-  int o = 0;
-  for (int j = lane; j < ui; j += 32)
-    o += min(max(p.accept_len[j], 0), p.q_off[j + 1] - p.q_off[j] - 1) + 1;
-  const int off = __reduce_add_sync(0xffffffffu, o);
-  for (int k = lane; k < a; k += 32) p.out_tokens[off + k] = p.draft_tokens[l0 + k];
-  if (lane == 0) {
-    p.out_offsets[ui] = off;
-    if (ui == p.B - 1) p.out_offsets[p.B] = off + a + 1;
-  }
-  const float u = p.uniforms[2 * n + 1];
   const float4* part = p.part2 + static_cast<size_t>(ui) * p.nseg2;
   const int per = (p.nseg2 + 31) >> 5;  // lane j owns segments [j per, (j + 1) per)
   const int s0 = lane * per;
@@ -665,18 +672,37 @@ __device__ __forceinline__ void descend(const SpecParams<CAP>& p, int ui, int a,
   // lane's total), so the walk below compares them all at once
   constexpr int kRun = 16;
   const bool in_regs = per <= kRun;
+  auto load_run = [&](int mode, float2 (&v)[kRun]) {
+#pragma unroll
+    for (int i = 0; i < kRun; ++i) {
+      const int sg = s0 + i;
+      v[i] = in_regs && i < per && sg < p.nseg2 ? __ldcg(reinterpret_cast<const float2*>(part + sg) + mode)
+                                                : make_float2(0.f, 0.f);
+    }
+  };
+  // every independent load first: the first mode's segment totals, the
+  // uniform, the accepted drafts and the earlier users' accept lengths
+  const int mode0 = residual ? 0 : 1;
+  float2 v[kRun];
+  load_run(mode0, v);
+  const float u = p.uniforms[2 * n + 1];
+  const int dtok = lane < a ? p.draft_tokens[l0 + lane] : 0;  // a <= L_i <= 31
+  int o = 0;
+  for (int j = lane; j < ui; j += 32)
+    o += min(max(p.accept_len[j], 0), p.q_off[j + 1] - p.q_off[j] - 1) + 1;
+  const int off = __reduce_add_sync(0xffffffffu, o);
+  if (lane < a) p.out_tokens[off + lane] = dtok;
+  if (lane == 0) {
+    p.counters[kCntUser2 + ui] = 0u;
+    p.out_offsets[ui] = off;
+    if (ui == p.B - 1) p.out_offsets[p.B] = off + a + 1;
+  }
   // mode 0: the residual; mode 1: p (the bonus position, or an empty residual)
-  for (int mode = residual ? 0 : 1; mode < 2; ++mode) {
+  for (int mode = mode0; mode < 2; ++mode) {
     FF pre[kRun];
     FF ls{0.f, 0.f};
     if (in_regs) {
-      float2 v[kRun];
-#pragma unroll
-      for (int i = 0; i < kRun; ++i) {
-        const int sg = s0 + i;
-        v[i] = i < per && sg < p.nseg2 ? __ldcg(reinterpret_cast<const float2*>(part + sg) + mode)
-                                       : make_float2(0.f, 0.f);
-      }
+      if (mode != mode0) load_run(mode, v);
 #pragma unroll
       for (int i = 0; i < kRun; ++i) {
         ls = ff_add(ls, FF{v[i].x, v[i].y});
@@ -686,8 +712,8 @@ __device__ __forceinline__ void descend(const SpecParams<CAP>& p, int ui, int a,
       for (int i = 0; i < per; ++i) {
         const int sg = s0 + i;
         if (sg < p.nseg2) {
-          const float2 v = __ldcg(reinterpret_cast<const float2*>(part + sg) + mode);
-          ls = ff_add(ls, FF{v.x, v.y});
+          const float2 w = __ldcg(reinterpret_cast<const float2*>(part + sg) + mode);
+          ls = ff_add(ls, FF{w.x, w.y});
         }
       }
     }
