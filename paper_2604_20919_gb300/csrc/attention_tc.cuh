@@ -546,38 +546,30 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
     uint8_t* xbuf = sK;  // every rank's K ring, drained once all ranks are here
     // slot of source rank `src` at receiving rank `dst`
     auto slot_of = [&](int src, int dst) { return (src < dst ? src : src - 1) * kSlot; };
-    // the whole O row in registers: one TMEM round trip serves the push and the merge
-    uint32_t o[kCh][32];
-    if (active && fin_ok) {
-      tc_fence_after();
-#pragma unroll
-      for (int cc = 0; cc < kCh; ++cc) tmem_ld32_async(tO + cc * 32 + lane_base, o[cc]);
-      tmem_wait_ld();
-#pragma unroll
-      for (int cc = 0; cc < kCh; ++cc) reg_fence32(o[cc]);
-    }
     cluster_arrive_release();
     cluster_wait_acquire();
-    if (active && fin_ok && valid) {
+    if (active && fin_ok) {
       for (int dst = 0; dst < C; ++dst)
-        if (dst != crank) dsmem_st_f32x2(dsmem_map(xbuf + slot_of(crank, dst), dst) + r * 8, fin_m, fin_l);
-      if (fin_l > 0.f) {
-#pragma unroll
-        for (int cc = 0; cc < kCh; ++cc) {
-          const int dst = cc % C;
-          if (dst == crank) continue;
+        if (dst != crank && valid) dsmem_st_f32x2(dsmem_map(xbuf + slot_of(crank, dst), dst) + r * 8, fin_m, fin_l);
+      tc_fence_after();
+#pragma unroll 1
+      for (int cc = 0; cc < kCh; ++cc) {
+        const int dst = cc % C;
+        if (dst == crank) continue;
+        uint32_t o[32];
+        tmem_ld32(tO + cc * 32 + lane_base, o);
+        if (valid && fin_l > 0.f) {
           const uint32_t base = dsmem_map(xbuf + slot_of(crank, dst), dst) + 1024 + (cc / C) * L::kChunkBytes;
 #pragma unroll
           for (int k = 0; k < 8; ++k)
-            dsmem_st_f32x4(base + (k * 128 + r) * 16, __uint_as_float(o[cc][4 * k]),
-                           __uint_as_float(o[cc][4 * k + 1]), __uint_as_float(o[cc][4 * k + 2]),
-                           __uint_as_float(o[cc][4 * k + 3]));
+            dsmem_st_f32x4(base + (k * 128 + r) * 16, __uint_as_float(o[4 * k]), __uint_as_float(o[4 * k + 1]),
+                           __uint_as_float(o[4 * k + 2]), __uint_as_float(o[4 * k + 3]));
         }
       }
     }
     cluster_arrive_release();
     cluster_wait_acquire();
-    if (active && fin_ok && valid && crank < kCh) {
+    if (active && fin_ok && crank < kCh) {
       const int t = rg / p.G, g = rg % p.G;
       float mx = fin_m;
       for (int s = 0; s < C; ++s)
@@ -592,12 +584,14 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
       }
       const float inv = l > 0.f ? 1.f / l : 0.f;
       __nv_bfloat16* orow = p.out + (static_cast<size_t>(U.q_off + t) * p.Hq + h * p.G + g) * D;
-#pragma unroll
-      for (int cc = 0; cc < kCh; ++cc) {
-        if (cc % C != crank) continue;
+      tc_fence_after();
+#pragma unroll 1
+      for (int cc = crank; cc < kCh; cc += C) {
+        uint32_t o[32];
+        tmem_ld32(tO + cc * 32 + lane_base, o);
         float acc[32];
 #pragma unroll
-        for (int k = 0; k < 32; ++k) acc[k] = w0 > 0.f ? w0 * __uint_as_float(o[cc][k]) : 0.f;
+        for (int k = 0; k < 32; ++k) acc[k] = w0 > 0.f ? w0 * __uint_as_float(o[k]) : 0.f;
         for (int s = 0; s < C; ++s) {
           if (s == crank) continue;
           const float2 ml = reinterpret_cast<const float2*>(xbuf + slot_of(s, crank))[r];
@@ -614,13 +608,15 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
             acc[4 * k + 3] += w * v.w;
           }
         }
-        uint4* dst = reinterpret_cast<uint4*>(orow + cc * 32);
+        if (valid) {
+          uint4* dst = reinterpret_cast<uint4*>(orow + cc * 32);
 #pragma unroll
-        for (int k = 0; k < 4; ++k)
-          dst[k] = make_uint4(pack_bf16x2(acc[8 * k] * inv, acc[8 * k + 1] * inv),
-                              pack_bf16x2(acc[8 * k + 2] * inv, acc[8 * k + 3] * inv),
-                              pack_bf16x2(acc[8 * k + 4] * inv, acc[8 * k + 5] * inv),
-                              pack_bf16x2(acc[8 * k + 6] * inv, acc[8 * k + 7] * inv));
+          for (int k = 0; k < 4; ++k)
+            dst[k] = make_uint4(pack_bf16x2(acc[8 * k] * inv, acc[8 * k + 1] * inv),
+                                pack_bf16x2(acc[8 * k + 2] * inv, acc[8 * k + 3] * inv),
+                                pack_bf16x2(acc[8 * k + 4] * inv, acc[8 * k + 5] * inv),
+                                pack_bf16x2(acc[8 * k + 6] * inv, acc[8 * k + 7] * inv));
+        }
       }
     }
     tc_fence_before();
