@@ -398,24 +398,27 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
       if (!ok) break;
       tc_fence_after();
       const uint32_t tSb = tS0 + b * kTcTile + lane_base;
-      // one tile's softmax over its first NC score columns (NC = 128, or 32
-      // for a last tile of at most two pages); false: a wait gave up
-      auto tile_softmax = [&](auto nc_tag) -> bool {
-        constexpr int NC = decltype(nc_tag)::value;
-        uint32_t sr[NC];
-        if constexpr (NC == 128) tmem_ld128(tSb, sr);
-        else tmem_ld32(tSb, sr);
-        // raw scores; the causal rule key <= C_i + t only bites near the end
-        // (columns past the tile's pages are keys past kv_end: masked too)
-        float s[NC];
+      if (active) {
+        // two passes over the tile's loaded columns in 32-column chunks (a
+        // small loop body: this code runs once per tile and per CTA, so its
+        // instruction fetch counts); the second pass overwrites S with P as it
+        // goes (P pairs of keys 32c..32c+31 land in columns 16c..16c+15, which
+        // this thread has already read)
+        const int nch = (tile_pages(j) * kPage + 31) / 32;
         float mr = -INFINITY;
-        const bool need_mask = key0 + NC - 1 > last_vis;
+#pragma unroll 1
+        for (int ch = 0; ch < nch; ++ch) {
+          uint32_t sr[32];
+          tmem_ld32(tSb + ch * 32, sr);
+          // raw scores; the causal rule key <= C_i + t only bites near the end
+          // (columns past the tile's pages are keys past kv_end: masked too)
+          const int kb = key0 + ch * 32;
+          const bool need_mask = kb + 31 > last_vis;
 #pragma unroll
-        for (int c = 0; c < NC; ++c) {
-          float v = __uint_as_float(sr[c]);
-          if (need_mask && key0 + c > last_vis) v = -INFINITY;
-          s[c] = v;
-          mr = fmaxf(mr, v);
+          for (int c = 0; c < 32; ++c) {
+            const float v = __uint_as_float(sr[c]);
+            mr = fmaxf(mr, need_mask && kb + c > last_vis ? -INFINITY : v);
+          }
         }
         const float mt = mr * sl2;  // tile maximum in log2 units (scale > 0)
         // lazy rescale: keep the old maximum unless this tile exceeds it by 2^8
@@ -427,10 +430,10 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
         }
         if (j > 0 && __any_sync(0xffffffffu, grow && factor != 1.f)) {
           // every earlier P V has to be done before O is touched
-          if (!__all_sync(0xffffffffu, mbar_wait(&pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1, p.status)))
-            return false;
+          ok = __all_sync(0xffffffffu, mbar_wait(&pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1, p.status));
+          if (!ok) break;
           tc_fence_after();
-#pragma unroll
+#pragma unroll 1
           for (int cc = 0; cc < D / 32; ++cc) {
             uint32_t o[32];
             tmem_ld32(tO + cc * 32 + lane_base, o);
@@ -441,29 +444,24 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
         }
         l *= factor;
         const float nb = m == -INFINITY ? 0.f : -m;
-        // P over the first NC / 2 columns of S[b] (already read); the P V that
-        // read this buffer two tiles ago completed before S[b] was written
-        constexpr int kPk = NC < 64 ? NC / 2 : 32;
+#pragma unroll 1
+        for (int ch = 0; ch < nch; ++ch) {
+          uint32_t sr[32];
+          tmem_ld32(tSb + ch * 32, sr);
+          const int kb = key0 + ch * 32;
+          const bool need_mask = kb + 31 > last_vis;
+          uint32_t pk[16];
 #pragma unroll
-        for (int hh = 0; hh < (NC + 63) / 64; ++hh) {
-          uint32_t pk[kPk];
-#pragma unroll
-          for (int c = 0; c < 2 * kPk; c += 2) {
-            const float p0 = fast_exp2(__fmaf_rn(s[hh * 64 + c], sl2, nb));
-            const float p1 = fast_exp2(__fmaf_rn(s[hh * 64 + c + 1], sl2, nb));
+          for (int c = 0; c < 32; c += 2) {
+            const float s0 = need_mask && kb + c > last_vis ? -INFINITY : __uint_as_float(sr[c]);
+            const float s1 = need_mask && kb + c + 1 > last_vis ? -INFINITY : __uint_as_float(sr[c + 1]);
+            const float p0 = fast_exp2(__fmaf_rn(s0, sl2, nb));
+            const float p1 = fast_exp2(__fmaf_rn(s1, sl2, nb));
             l += p0 + p1;
             pk[c >> 1] = pack_bf16x2(p0, p1);
           }
-          if constexpr (kPk == 32) tmem_st32(tSb + hh * 32, pk);
-          else tmem_st16(tSb + hh * 32, pk);
+          tmem_st16(tSb + ch * 16, pk);
         }
-        return true;
-      };
-      if (active) {
-        const bool done = tile_pages(j) * kPage <= 32 ? tile_softmax(std::integral_constant<int, 32>{})
-                                                      : tile_softmax(std::integral_constant<int, kTcTile>{});
-        ok = done;
-        if (!ok) break;
       } else {
         uint32_t pk[32];
 #pragma unroll
