@@ -43,10 +43,11 @@ constexpr int kRegThreads = 256;
 constexpr int kRegWarps = kRegThreads / 32;
 
 // Row statistics of one verify position, relative to integer references:
-// sz = sum_v 2^(z_v log2 e - cz), sw likewise for the draft row; sz / sw, the
-// scale of q against p in the residual, split into two floats.
+// sz = sum_v 2^(z_v log2 e - cz), sw likewise for the draft row, each a
+// float-float pair; sz / sw, the scale of q against p in the residual, split
+// into two floats.
 struct SpecStat {
-  double sz, sw;
+  float szh, szl, swh, swl;
   int cz, cw;
   float khi, klo;
 };
@@ -506,14 +507,18 @@ __device__ __forceinline__ void decide_from_sums(const SpecParams<CAP>& p, int u
   const int n = q0 + t;
   const bool has_q = t < Li;
   {
+    // float-float throughout (FP64 is slow on this part): the acceptance
+    // products carry ~2^-45 relative error, far inside the 1e-6 band
     SpecStat st;
-    st.sz = static_cast<double>(az.s.hi) + static_cast<double>(az.s.lo);
+    st.szh = az.s.hi;
+    st.szl = az.s.lo;
     st.cz = az.c;
-    st.sw = 0.0;
+    st.swh = st.swl = 0.f;
     st.cw = kEmptyRef;
     st.khi = st.klo = 0.f;
     float pd = 0.f, qd = 0.f;
     unsigned char flag = 0;
+    const float u = p.uniforms[2 * n];
     if (has_q && SP) {
       // sparse payload: q(d) is given; the residual scales q by sz, kept as
       // a float-float pair
@@ -521,16 +526,17 @@ __device__ __forceinline__ void decide_from_sums(const SpecParams<CAP>& p, int u
       st.klo = az.s.lo;
       if (zd == zd) {
         const float ez = ex2_ref(zd, st.cz);
-        const double q_d = exp(static_cast<double>(logq));
-        pd = ez * (1.f / static_cast<float>(st.sz));
-        qd = static_cast<float>(q_d);
+        const float q_d = expf(logq);
+        pd = __fdividef(ez, az.s.hi);
+        qd = q_d;
         // u * q(d) < p(d) = ez / sz, i.e. u * q(d) * sz < ez
-        flag = static_cast<double>(p.uniforms[2 * n]) * q_d * st.sz < static_cast<double>(ez) ? 1 : 0;
+        flag = ff_gt(FF{ez, 0.f}, ff_mul_f(ff_mul_f(az.s, u), q_d)) ? 1 : 0;
       } else {
         atomicOr(p.status, kDevErrBadToken);
       }
     } else if (has_q) {
-      st.sw = static_cast<double>(aw.s.hi) + static_cast<double>(aw.s.lo);
+      st.swh = aw.s.hi;
+      st.swl = aw.s.lo;
       st.cw = aw.c;
       // sz / sw in float-float: q1 = zh / wh, then the remainder's quotient
       const float q1 = __fdiv_rn(az.s.hi, aw.s.hi);
@@ -542,11 +548,10 @@ __device__ __forceinline__ void decide_from_sums(const SpecParams<CAP>& p, int u
       if (zd == zd && wd == wd) {
         const float ez = ex2_ref(zd, st.cz);
         const float ew = ex2_ref(wd, st.cw);
-        pd = ez * (1.f / static_cast<float>(st.sz));
-        qd = ew * (1.f / static_cast<float>(st.sw));
-        // u * q(d) < p(d), i.e. u * ew * sz < ez * sw (products in fp64, no division)
-        flag = static_cast<double>(p.uniforms[2 * n]) * static_cast<double>(ew) * st.sz <
-                       static_cast<double>(ez) * st.sw ? 1 : 0;
+        pd = __fdividef(ez, az.s.hi);
+        qd = __fdividef(ew, aw.s.hi);
+        // u * q(d) < p(d), i.e. u * ew * sz < ez * sw (no division)
+        flag = ff_gt(ff_mul_f(aw.s, ez), ff_mul_f(ff_mul_f(az.s, u), ew)) ? 1 : 0;
       } else {
         atomicOr(p.status, kDevErrBadToken);
       }
