@@ -413,14 +413,8 @@ def run_dipsd(args):
     emitted = int(outs[1][-1].item())
     units = emitted * n_steps
     total_ms = ms_step * n_steps
-    if world > 1:
-        tt = torch.tensor([total_ms, units, float(np.sum(e2e_ms))], dtype=torch.float64, device=dev)
-        mx = tt.clone()
-        dist.all_reduce(mx, op=dist.ReduceOp.MAX)
-        dist.all_reduce(tt, op=dist.ReduceOp.SUM)
-        total_ms_max, units_all, e2e_max = float(mx[0]), float(tt[1]), float(mx[2])
-    else:
-        total_ms_max, units_all, e2e_max = total_ms, float(units), float(np.sum(e2e_ms))
+    from paper_2604_20919_gb300.shard import aggregate_timing
+    total_ms_max, units_all, e2e_max = aggregate_timing(total_ms, units, float(np.sum(e2e_ms)), device=dev)
     if rank != 0:
         if world > 1:
             dist.destroy_process_group()
