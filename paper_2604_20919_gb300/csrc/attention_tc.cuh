@@ -28,11 +28,12 @@
 //               issuing thread, not the tensor core, is what bounds the
 //               tile rate, so tiles are as long as the rings allow.
 //   warps 2..5  one query row per thread (TMEM lane = row): put the Q row
-//               in TMEM, then per tile load S[b] with
-//               tcgen05.ld, causal mask, online softmax in log2 units with a
-//               lazy rescale (O in TMEM is rescaled only when a row maximum
-//               grows by more than 2^8), write P as bf16 pairs into the first
-//               32 columns of S[b] with tcgen05.st, and finally read O back.
+//               in TMEM, then per tile read S[b] in 32-column chunks with
+//               tcgen05.ld twice (tile maximum, then P), causal mask, online
+//               softmax in log2 units with a lazy rescale (O in TMEM is
+//               rescaled only when a row maximum grows by more than 2^8),
+//               write P as bf16 pairs into the first 64 columns of S[b] with
+//               tcgen05.st, and finally read O back.
 // KV append (p.new_k set): the T_i new rows are not read from the cache.
 // The producer patches them into every K/V tile that covers positions
 // C_i .. C_i + T_i - 1 once the tile has landed, and signals the tile on

@@ -4,7 +4,6 @@
 #pragma once
 
 #include <cstdint>
-#include <type_traits>
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
