@@ -21,7 +21,7 @@ position t):
      is drawn from p_{L_i}.
   5. emitted_i = d_1 .. d_{a_i}, then that extra token.
 
-Readings where the method leaves a choice (each listed in the design doc):
+Readings where the method leaves a choice:
   * uniforms are inputs: uniforms[n] = (u_acc, u_res) for verify position n;
   * sampling is an inverse CDF in ascending token order: the smallest k with
     cumsum(w)[k] > u * sum(w); if rounding leaves none, the last k with w_k > 0;
