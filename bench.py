@@ -44,7 +44,8 @@ def parse_args():
     ap.add_argument("--impl", choices=["dipsd", "reference"], default="dipsd")
     ap.add_argument("--workload", type=int, default=2, help="workload id (2 = the headline batch)")
     ap.add_argument("--seed", type=int, default=0)
-    ap.add_argument("--cpu-seconds", type=float, default=10.0, help="budget of the CPU oracle baseline")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0,
+                    help="budget of the CPU oracle baseline (0: skip it, for the large non-headline workloads)")
     return ap.parse_args()
 
 
@@ -479,7 +480,7 @@ def run_dipsd(args):
         "gpu_launches": int(launches),
         "clocks": clocks,
     }
-    if world == 1:
+    if world == 1 and args.cpu_seconds > 0:
         line["cpu_baseline"] = cpu_baseline(b, args.cpu_seconds)
     print(json.dumps(line), flush=True)
     if world > 1:
