@@ -89,7 +89,9 @@ constexpr int kTcStages = TcSmem<128>::kStages;
 // tm_k: 4-D {64 columns, 16 rows, heads, blocks}, one 64-column half of a
 // page per box; tm_v: 5-D {64 columns, 16 rows, halves, heads, blocks}, a
 // whole page per box.
-template <int D, int CAP>
+// PERSIST: the grid is smaller than the item count and each CTA walks
+// several items; otherwise every CTA runs exactly one (the single-pass code).
+template <int D, int CAP, bool PERSIST>
 __global__ void __launch_bounds__(kTcThreads, 1)
 verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __grid_constant__ CUtensorMap tm_k,
                            const __grid_constant__ CUtensorMap tm_v) {
@@ -114,26 +116,34 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
   uint64_t* v_patch = k_patch + S;   // [S]
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(v_patch + S);
 
-  // ---- work item
-  const int item = blockIdx.x;
-  const int ui = find_user<CAP>(p.item_off, p.B, item);
-  const AttnUser U = p.u[ui];
-  int local = item - p.item_off[ui];
-  const int split = local % U.nsplit;
-  local /= U.nsplit;
-  const int h = local % p.Hkv;
-  const int rb = local / p.Hkv;
-  const int M = p.G * U.T;
-  const int row0 = rb * 128;
-  const int kv_begin = split * U.split_len;
-  const int kv_end = min(kv_begin + U.split_len, U.kv_len);
-  const int ntiles = max(0, (kv_end - kv_begin + kTcTile - 1) / kTcTile);  // 0: an empty split
-  // Splits start on a page.  A split's last tile holds only the pages up to
-  // kv_end: only those are loaded, multiplied (Q K^T with N = 16 per page,
-  // one P V step per page) and run through the softmax.
-  const int split_pages_n = (kv_end + kPage - 1) / kPage - kv_begin / kPage;
+  // ---- work items: this CTA takes blockIdx.x, blockIdx.x + gridDim.x, ...
+  // (one item when the grid has an item per CTA).  Every role walks the same
+  // items in the same order; ring slots and barrier phases run on across
+  // items (global tile index g0 + j).
+  int ui, split, h, rb, M, row0, kv_begin, kv_end, ntiles, split_pages_n;
+  AttnUser U;
+  auto set_item = [&](int item) {
+    ui = find_user<CAP>(p.item_off, p.B, item);
+    U = p.u[ui];
+    int local = item - p.item_off[ui];
+    split = local % U.nsplit;
+    local /= U.nsplit;
+    h = local % p.Hkv;
+    rb = local / p.Hkv;
+    M = p.G * U.T;
+    row0 = rb * 128;
+    kv_begin = split * U.split_len;
+    kv_end = min(kv_begin + U.split_len, U.kv_len);
+    ntiles = max(0, (kv_end - kv_begin + kTcTile - 1) / kTcTile);  // 0: an empty split
+    // Splits start on a page.  A split's last tile holds only the pages up
+    // to kv_end: only those are loaded, multiplied (Q K^T with N = 16 per
+    // page, one P V step per page) and run through the softmax.
+    split_pages_n = (kv_end + kPage - 1) / kPage - kv_begin / kPage;
+  };
+  set_item(blockIdx.x);
   auto tile_pages = [&](int j) { return min(kTcTile / kPage, split_pages_n - j * (kTcTile / kPage)); };
-  // tile j holds new (appended) rows: keys [max(key0, C_i), min(key0 + 128, kv_end))
+  // tile j holds new (appended) rows: keys [max(key0, C_i), min(key0 + 128, kv_end)).
+  // The patch barriers are single-use: a launch that appends runs one item per CTA.
   auto patched = [&](int j) {
     const int key0 = kv_begin + j * kTcTile;
     return p.new_k != nullptr && max(key0, U.ctx) < min(key0 + kTcTile, kv_end);
@@ -183,13 +193,6 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
     // ------------------------------------------------------------ producer
     // Page ids come from the block table 32 at a time (one per lane, one
     // group of 8 tiles ahead) so no TMA waits on a dependent global load.
-    const int* bt = p.block_table + static_cast<size_t>(U.bt_row) * p.max_blocks;
-    const int n_pages = (kv_end + kPage - 1) / kPage;  // pages of this split end here
-    const int page_base = kv_begin / kPage;
-    auto fetch = [&](int group) {
-      const int page = page_base + group * 32 + lane;
-      return page < n_pages ? __ldg(bt + page) : p.num_blocks;  // past the end: never requested
-    };
     constexpr int kPages = kTcTile / kPage;
     constexpr int kTilesPerGroup = 32 / kPages;
     constexpr int kKBoxes = kPages * kHalves;  // K boxes per tile; V: kPages
@@ -198,85 +201,110 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
     const int vb = lane - kKBoxes;
     const int my_pg = lane < kKBoxes ? kb / kHalves : (vb & (kPages - 1));
     const int my_hf = kb % kHalves;
-    int cur = fetch(0);
-    int nxt = fetch(1);
-    int issued = 0;
-    for (int j = 0; j < ntiles; ++j) {
-      const int st = j % S;
-      if (j % kTilesPerGroup == 0 && j > 0) {
-        cur = nxt;
-        nxt = fetch(j / kTilesPerGroup + 1);
-      }
-      const int bk = __shfl_sync(0xffffffffu, cur, (j % kTilesPerGroup) * kPages + my_pg);
-      const uint32_t ph = ((j / S) - 1) & 1;
-      const uint32_t koff = st * L::kTileBytes + my_hf * (kTcTile * 128) + my_pg * (kPage * 128);
-      const uint32_t voff = st * L::kTileBytes + my_pg * L::kPageBytes;
-      const int tp = tile_pages(j);  // pages of this tile (kPages except in a split's last tile)
-      // K tile
-      bool go = true;
-      if (j >= S && lane == 0) go = mbar_wait(&k_empty[st], ph, p.status);
-      if (!__shfl_sync(0xffffffffu, go, 0)) break;
-      if (lane == 0) mbar_arrive_expect_tx(&k_full[st], tp * L::kPageBytes);
-      __syncwarp();
-      if (lane < kKBoxes && my_pg < tp) tma_load_4d(sK + koff, &tm_k, my_hf * 64, 0, h, bk, &k_full[st]);
-      // V tile
-      if (j >= S && lane == 0) go = mbar_wait(&v_empty[st], ph, p.status);
-      if (!__shfl_sync(0xffffffffu, go, 0)) break;
-      if (lane == 0) mbar_arrive_expect_tx(&v_full[st], tp * L::kPageBytes);
-      __syncwarp();
-      if (lane >= kKBoxes && lane < kKBoxes + kPages && my_pg < tp)
-        tma_load_5d(sV + voff, &tm_v, 0, 0, 0, h, bk, &v_full[st]);
-      ++issued;
-      if (patched(j)) {
-        // the appended rows of this tile, straight from the input, over what
-        // the pages held (generic writes, then a proxy fence for the MMA)
-        const int key0 = kv_begin + j * kTcTile;
-        const int lo = max(key0, U.ctx), hi = min(key0 + kTcTile, kv_end);
-        const int n16 = (hi - lo) * (D / 8);
-        go = true;
-        if (lane == 0) go = mbar_wait(&k_full[st], (j / S) & 1, p.status);
-        if (!__shfl_sync(0xffffffffu, go, 0)) break;
-        for (int e = lane; e < n16; e += 32) {
-          const int key = lo + e / (D / 8), c = e % (D / 8), r = key - key0;
-          const uint4 v = __ldg(reinterpret_cast<const uint4*>(
-              p.new_k + (static_cast<size_t>(U.q_off + key - U.ctx) * p.Hkv + h) * D) + c);
-          *reinterpret_cast<uint4*>(sK + st * L::kTileBytes + (c >> 3) * (kTcTile * 128) + r * 128 +
-                                    (((c & 7) ^ (r & 7)) << 4)) = v;
+    int issued = 0;  // tiles issued over all items (the global tile index of the next)
+    bool alive = true;
+    for (int item = blockIdx.x, n = 0; (PERSIST || n == 0) && item < p.n_items && alive; item += gridDim.x, ++n) {
+      if (n > 0) set_item(item);
+      const int g0 = issued;
+      const int* bt = p.block_table + static_cast<size_t>(U.bt_row) * p.max_blocks;
+      const int n_pages = (kv_end + kPage - 1) / kPage;  // pages of this split end here
+      const int page_base = kv_begin / kPage;
+      auto fetch = [&](int group) {
+        const int page = page_base + group * 32 + lane;
+        return page < n_pages ? __ldg(bt + page) : p.num_blocks;  // past the end: never requested
+      };
+      int cur = fetch(0);
+      int nxt = fetch(1);
+      for (int j = 0; j < ntiles; ++j) {
+        const int gj = g0 + j;
+        const int st = gj % S;
+        if (j % kTilesPerGroup == 0 && j > 0) {
+          cur = nxt;
+          nxt = fetch(j / kTilesPerGroup + 1);
         }
-        fence_proxy_async_smem();
+        const int bk = __shfl_sync(0xffffffffu, cur, (j % kTilesPerGroup) * kPages + my_pg);
+        const uint32_t ph = ((gj / S) - 1) & 1;
+        const uint32_t koff = st * L::kTileBytes + my_hf * (kTcTile * 128) + my_pg * (kPage * 128);
+        const uint32_t voff = st * L::kTileBytes + my_pg * L::kPageBytes;
+        const int tp = tile_pages(j);  // pages of this tile (kPages except in a split's last tile)
+        // K tile
+        bool go = true;
+        if (gj >= S && lane == 0) go = mbar_wait(&k_empty[st], ph, p.status);
+        if (!__shfl_sync(0xffffffffu, go, 0)) {
+          alive = false;
+          break;
+        }
+        if (lane == 0) mbar_arrive_expect_tx(&k_full[st], tp * L::kPageBytes);
         __syncwarp();
-        if (lane == 0) mbar_arrive(&k_patch[st]);
-        if (lane == 0) go = mbar_wait(&v_full[st], (j / S) & 1, p.status);
-        if (!__shfl_sync(0xffffffffu, go, 0)) break;
-        for (int e = lane; e < n16; e += 32) {
-          const int key = lo + e / (D / 8), c = e % (D / 8), r = key - key0;
-          const int r16 = r % kPage;
-          const uint4 v = __ldg(reinterpret_cast<const uint4*>(
-              p.new_v + (static_cast<size_t>(U.q_off + key - U.ctx) * p.Hkv + h) * D) + c);
-          *reinterpret_cast<uint4*>(sV + st * L::kTileBytes + (r / kPage) * L::kPageBytes + (c >> 3) * (kPage * 128) +
-                                    r16 * 128 + (((c & 7) ^ (r16 & 7)) << 4)) = v;
+        if (lane < kKBoxes && my_pg < tp) tma_load_4d(sK + koff, &tm_k, my_hf * 64, 0, h, bk, &k_full[st]);
+        // V tile
+        if (gj >= S && lane == 0) go = mbar_wait(&v_empty[st], ph, p.status);
+        if (!__shfl_sync(0xffffffffu, go, 0)) {
+          alive = false;
+          break;
         }
-        fence_proxy_async_smem();
+        if (lane == 0) mbar_arrive_expect_tx(&v_full[st], tp * L::kPageBytes);
         __syncwarp();
-        if (lane == 0) mbar_arrive(&v_patch[st]);
-      }
-    }
-    // state update: the last split of the first row block writes the user's
-    // new rows of head h into the pages
-    if (p.new_k != nullptr && rb == 0 && split == U.nsplit - 1) {
-      const int n16 = U.T * (D / 8);
-      for (int e = lane; e < n16; e += 32) {
-        const int tt = e / (D / 8), c = e % (D / 8);
-        const int pos = U.ctx + tt;
-        const int blk = __ldg(bt + pos / kPage);
-        if (blk < 0 || blk >= p.num_blocks) {
-          atomicOr(p.status, kDevErrBadBlock);
-          continue;
+        if (lane >= kKBoxes && lane < kKBoxes + kPages && my_pg < tp)
+          tma_load_5d(sV + voff, &tm_v, 0, 0, 0, h, bk, &v_full[st]);
+        ++issued;
+        if (patched(j)) {
+          // the appended rows of this tile, straight from the input, over what
+          // the pages held (generic writes, then a proxy fence for the MMA)
+          const int key0 = kv_begin + j * kTcTile;
+          const int lo = max(key0, U.ctx), hi = min(key0 + kTcTile, kv_end);
+          const int n16 = (hi - lo) * (D / 8);
+          go = true;
+          if (lane == 0) go = mbar_wait(&k_full[st], (gj / S) & 1, p.status);
+          if (!__shfl_sync(0xffffffffu, go, 0)) {
+            alive = false;
+            break;
+          }
+          for (int e = lane; e < n16; e += 32) {
+            const int key = lo + e / (D / 8), c = e % (D / 8), r = key - key0;
+            const uint4 v = __ldg(reinterpret_cast<const uint4*>(
+                p.new_k + (static_cast<size_t>(U.q_off + key - U.ctx) * p.Hkv + h) * D) + c);
+            *reinterpret_cast<uint4*>(sK + st * L::kTileBytes + (c >> 3) * (kTcTile * 128) + r * 128 +
+                                      (((c & 7) ^ (r & 7)) << 4)) = v;
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&k_patch[st]);
+          if (lane == 0) go = mbar_wait(&v_full[st], (gj / S) & 1, p.status);
+          if (!__shfl_sync(0xffffffffu, go, 0)) {
+            alive = false;
+            break;
+          }
+          for (int e = lane; e < n16; e += 32) {
+            const int key = lo + e / (D / 8), c = e % (D / 8), r = key - key0;
+            const int r16 = r % kPage;
+            const uint4 v = __ldg(reinterpret_cast<const uint4*>(
+                p.new_v + (static_cast<size_t>(U.q_off + key - U.ctx) * p.Hkv + h) * D) + c);
+            *reinterpret_cast<uint4*>(sV + st * L::kTileBytes + (r / kPage) * L::kPageBytes +
+                                      (c >> 3) * (kPage * 128) + r16 * 128 + (((c & 7) ^ (r16 & 7)) << 4)) = v;
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&v_patch[st]);
         }
-        const size_t dst = ((static_cast<size_t>(blk) * p.Hkv + h) * kPage + pos % kPage) * D;
-        const size_t src = (static_cast<size_t>(U.q_off + tt) * p.Hkv + h) * D;
-        reinterpret_cast<uint4*>(p.k_cache + dst)[c] = __ldg(reinterpret_cast<const uint4*>(p.new_k + src) + c);
-        reinterpret_cast<uint4*>(p.v_cache + dst)[c] = __ldg(reinterpret_cast<const uint4*>(p.new_v + src) + c);
+      }
+      // state update: the last split of the first row block writes the user's
+      // new rows of head h into the pages
+      if (alive && p.new_k != nullptr && rb == 0 && split == U.nsplit - 1) {
+        const int n16 = U.T * (D / 8);
+        for (int e = lane; e < n16; e += 32) {
+          const int tt = e / (D / 8), c = e % (D / 8);
+          const int pos = U.ctx + tt;
+          const int blk = __ldg(bt + pos / kPage);
+          if (blk < 0 || blk >= p.num_blocks) {
+            atomicOr(p.status, kDevErrBadBlock);
+            continue;
+          }
+          const size_t dst = ((static_cast<size_t>(blk) * p.Hkv + h) * kPage + pos % kPage) * D;
+          const size_t src = (static_cast<size_t>(U.q_off + tt) * p.Hkv + h) * D;
+          reinterpret_cast<uint4*>(p.k_cache + dst)[c] = __ldg(reinterpret_cast<const uint4*>(p.new_k + src) + c);
+          reinterpret_cast<uint4*>(p.v_cache + dst)[c] = __ldg(reinterpret_cast<const uint4*>(p.new_v + src) + c);
+        }
       }
     }
     // copies still in flight must land before the CTA can exit
@@ -292,238 +320,255 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
       constexpr uint32_t kIdPV = idesc_bf16_f32(128, D, false, true);
       const uint32_t k_addr = smem_addr(sK);
       const uint32_t v_addr = smem_addr(sV);
-      bool ok = mbar_wait(q_ready, 0, p.status);
-      int jq = 0, jp = 0;  // next Q K^T, next P V
-      uint64_t idle_since = 0;
-      uint32_t idle_polls = 0;
-      while (ok && jp < ntiles) {
-        bool did = false;
-        // S[jq & 1] is free once P V of tile jq - 2 has been issued (the
-        // tensor core runs one thread's MMAs in issue order)
-        if (jq < ntiles && jp >= jq - 1 &&
-            (patched(jq) ? mbar_test_wait(&k_patch[jq % S], 0) : mbar_test_wait(&k_full[jq % S], (jq / S) & 1))) {
-          tc_fence_after();
-          const uint32_t kt = k_addr + (jq % S) * L::kTileBytes;
-          // N = 16 keys per loaded page
-          const uint32_t id_qk = jq + 1 < ntiles ? kIdQK : idesc_bf16_f32(128, tile_pages(jq) * kPage, false, false);
+      bool ok = true;
+      int g0 = 0;  // global index of the item's first tile
+      for (int item = blockIdx.x, n = 0; (PERSIST || n == 0) && item < p.n_items && ok; item += gridDim.x, ++n) {
+        if (n > 0) set_item(item);
+        // Q of this item is in TMEM (written once the previous item's products were done)
+        ok = mbar_wait(q_ready, n & 1, p.status);
+        int jq = 0, jp = 0;  // next Q K^T, next P V (within the item)
+        uint64_t idle_since = 0;
+        uint32_t idle_polls = 0;
+        while (ok && jp < ntiles) {
+          bool did = false;
+          const int gq = g0 + jq, gp = g0 + jp;
+          // S[gq & 1] is free once P V of tile gq - 2 has been issued (the
+          // tensor core runs one thread's MMAs in issue order)
+          if (jq < ntiles && jp >= jq - 1 &&
+              (patched(jq) ? mbar_test_wait(&k_patch[gq % S], 0) : mbar_test_wait(&k_full[gq % S], (gq / S) & 1))) {
+            tc_fence_after();
+            const uint32_t kt = k_addr + (gq % S) * L::kTileBytes;
+            // N = 16 keys per loaded page
+            const uint32_t id_qk = jq + 1 < ntiles ? kIdQK : idesc_bf16_f32(128, tile_pages(jq) * kPage, false, false);
 #pragma unroll
-          for (int kk = 0; kk < D / 16; ++kk) {
-            const uint64_t bd = smem_desc_sw128(kt + (kk >> 2) * (kTcTile * 128) + (kk & 3) * 32, 0, 1024);
-            tc_mma_ts(tS0 + (jq & 1) * kTcTile, tQ + kk * 8, bd, id_qk, kk > 0 ? 1u : 0u);
+            for (int kk = 0; kk < D / 16; ++kk) {
+              const uint64_t bd = smem_desc_sw128(kt + (kk >> 2) * (kTcTile * 128) + (kk & 3) * 32, 0, 1024);
+              tc_mma_ts(tS0 + (gq & 1) * kTcTile, tQ + kk * 8, bd, id_qk, kk > 0 ? 1u : 0u);
+            }
+            tc_commit(&s_full[gq & 1]);
+            tc_commit(&k_empty[gq % S]);
+            ++jq;
+            did = true;
           }
-          tc_commit(&s_full[jq & 1]);
-          tc_commit(&k_empty[jq % S]);
-          ++jq;
-          did = true;
-        }
-        if (jp < jq && mbar_test_wait(&p_full[jp & 1], (jp >> 1) & 1) &&
-            (patched(jp) ? mbar_test_wait(&v_patch[jp % S], 0) : mbar_test_wait(&v_full[jp % S], (jp / S) & 1))) {
-          tc_fence_after();
-          const uint32_t vt = v_addr + (jp % S) * L::kTileBytes;
-          const uint32_t pt = tS0 + (jp & 1) * kTcTile;  // P: 64 columns of bf16 pairs
-          const int np = tile_pages(jp);
+          if (jp < jq && mbar_test_wait(&p_full[gp & 1], (gp >> 1) & 1) &&
+              (patched(jp) ? mbar_test_wait(&v_patch[gp % S], 0) : mbar_test_wait(&v_full[gp % S], (gp / S) & 1))) {
+            tc_fence_after();
+            const uint32_t vt = v_addr + (gp % S) * L::kTileBytes;
+            const uint32_t pt = tS0 + (gp & 1) * kTcTile;  // P: 64 columns of bf16 pairs
+            const int np = tile_pages(jp);
 #pragma unroll
-          for (int kk = 0; kk < kTcTile / kPage; ++kk) {
-            if (kk >= np) break;
-            // MN-major V page: 64-column halves kPage * 128 bytes apart
-            // (leading offset), 8-key groups 1024 bytes apart (stride offset)
-            const uint64_t bd = smem_desc_sw128(vt + kk * L::kPageBytes, kPage * 128, 1024);
-            tc_mma_ts(tO, pt + kk * 8, bd, kIdPV, (jp > 0 || kk > 0) ? 1u : 0u);
+            for (int kk = 0; kk < kTcTile / kPage; ++kk) {
+              if (kk >= np) break;
+              // MN-major V page: 64-column halves kPage * 128 bytes apart
+              // (leading offset), 8-key groups 1024 bytes apart (stride offset);
+              // the item's first product overwrites O
+              const uint64_t bd = smem_desc_sw128(vt + kk * L::kPageBytes, kPage * 128, 1024);
+              tc_mma_ts(tO, pt + kk * 8, bd, kIdPV, (jp > 0 || kk > 0) ? 1u : 0u);
+            }
+            tc_commit(&pv_done[gp & 1]);
+            tc_commit(&v_empty[gp % S]);
+            ++jp;
+            did = true;
           }
-          tc_commit(&pv_done[jp & 1]);
-          tc_commit(&v_empty[jp % S]);
-          ++jp;
-          did = true;
-        }
-        // the wait stays bounded, but the timer is read once per 256 idle
-        // polls: a %globaltimer read costs far more than a test_wait
-        if (did) {
-          idle_polls = 0;
-          idle_since = 0;
-        } else if ((++idle_polls & 255u) == 0) {
-          const uint64_t now = global_timer_ns();
-          if (idle_since == 0) {
-            idle_since = now;
-          } else if (now - idle_since > kWaitLimitNs) {
-            atomicOr(p.status, kDevErrWaitTimeout);
-            ok = false;
+          // the wait stays bounded, but the timer is read once per 256 idle
+          // polls: a %globaltimer read costs far more than a test_wait
+          if (did) {
+            idle_polls = 0;
+            idle_since = 0;
+          } else if ((++idle_polls & 255u) == 0) {
+            const uint64_t now = global_timer_ns();
+            if (idle_since == 0) {
+              idle_since = now;
+            } else if (now - idle_since > kWaitLimitNs) {
+              atomicOr(p.status, kDevErrWaitTimeout);
+              ok = false;
+            }
           }
         }
+        tc_commit(o_final);
+        g0 += ntiles;
       }
-      tc_commit(o_final);
     }
   } else {
     // ----------------------------------------- softmax / epilogue (row per thread)
     const int quad = warp & 3;
     const int r = quad * 32 + lane;  // row within the block == TMEM lane
-    const int rg = row0 + r;         // row within the user
-    const bool valid = rg < M;
-    const int t = rg / p.G, g = rg % p.G;
     const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;
-
-    // Q row -> TMEM lane r as bf16 pairs (column c holds elements 2c, 2c+1);
-    // padding rows are zero
-    {
-      const uint4* qrow =
-          reinterpret_cast<const uint4*>(p.q + (static_cast<size_t>(U.q_off + t) * p.Hq + h * p.G + g) * D);
-#pragma unroll
-      for (int cc = 0; cc < D / 64; ++cc) {
-        uint32_t w[32];
-#pragma unroll
-        for (int c = 0; c < 8; ++c) {
-          uint4 v = make_uint4(0, 0, 0, 0);
-          if (valid) v = __ldg(qrow + cc * 8 + c);
-          w[4 * c] = v.x;
-          w[4 * c + 1] = v.y;
-          w[4 * c + 2] = v.z;
-          w[4 * c + 3] = v.w;
-        }
-        tmem_st32(tQ + cc * 32 + lane_base, w);
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(q_ready);
-    }
-
-    const int last_vis = min(U.ctx + t, kv_end - 1);  // last key of this row in this split
-    // warps whose 32 rows are all padding write zero P, so every lane of P
-    // the tensor core reads is defined
-    const bool active = row0 + quad * 32 < M;
-    const float sl2 = p.scale_log2;
-    float m = -INFINITY, l = 0.f;
     bool ok = true;
-    for (int j = 0; j < ntiles; ++j) {
-      const int b = j & 1, st = j % S;
-      const int key0 = kv_begin + j * kTcTile;
-      ok = __all_sync(0xffffffffu, mbar_wait(&s_full[b], (j >> 1) & 1, p.status));
-      if (!ok) break;
-      tc_fence_after();
-      const uint32_t tSb = tS0 + b * kTcTile + lane_base;
-      if (active) {
-        // two passes over the tile's loaded columns in 32-column chunks (a
-        // small loop body: this code runs once per tile and per CTA, so its
-        // instruction fetch counts); the second pass overwrites S with P as it
-        // goes (P pairs of keys 32c..32c+31 land in columns 16c..16c+15, which
-        // this thread has already read)
-        const int nch = (tile_pages(j) * kPage + 31) / 32;
-        float mr = -INFINITY;
-#pragma unroll 1
-        for (int ch = 0; ch < nch; ++ch) {
-          uint32_t sr[32];
-          tmem_ld32(tSb + ch * 32, sr);
-          // raw scores; the causal rule key <= C_i + t only bites near the end
-          // (columns past the tile's pages are keys past kv_end: masked too)
-          const int kb = key0 + ch * 32;
-          const bool need_mask = kb + 31 > last_vis;
+    int g0 = 0;  // global index of the item's first tile
+    for (int item = blockIdx.x, n = 0; (PERSIST || n == 0) && item < p.n_items && ok; item += gridDim.x, ++n) {
+      if (n > 0) set_item(item);
+      const int rg = row0 + r;  // row within the user
+      const bool valid = rg < M;
+      const int t = rg / p.G, g = rg % p.G;
+
+      // Q row -> TMEM lane r as bf16 pairs (column c holds elements 2c, 2c+1);
+      // padding rows are zero.  The previous item's products are done (its
+      // o_final was waited for), so its Q is no longer read.
+      {
+        tc_fence_after();
+        const uint4* qrow =
+            reinterpret_cast<const uint4*>(p.q + (static_cast<size_t>(U.q_off + t) * p.Hq + h * p.G + g) * D);
 #pragma unroll
-          for (int c = 0; c < 32; ++c) {
-            const float v = __uint_as_float(sr[c]);
-            mr = fmaxf(mr, need_mask && kb + c > last_vis ? -INFINITY : v);
+        for (int cc = 0; cc < D / 64; ++cc) {
+          uint32_t w[32];
+#pragma unroll
+          for (int c = 0; c < 8; ++c) {
+            uint4 v = make_uint4(0, 0, 0, 0);
+            if (valid) v = __ldg(qrow + cc * 8 + c);
+            w[4 * c] = v.x;
+            w[4 * c + 1] = v.y;
+            w[4 * c + 2] = v.z;
+            w[4 * c + 3] = v.w;
           }
+          tmem_st32(tQ + cc * 32 + lane_base, w);
         }
-        const float mt = mr * sl2;  // tile maximum in log2 units (scale > 0)
-        // lazy rescale: keep the old maximum unless this tile exceeds it by 2^8
-        const bool grow = m == -INFINITY ? (mt > -INFINITY) : (mt > m + kRescaleThreshold);
-        float factor = 1.f;
-        if (grow) {
-          factor = m == -INFINITY ? 1.f : fast_exp2(m - mt);
-          m = mt;
-        }
-        if (j > 0 && __any_sync(0xffffffffu, grow && factor != 1.f)) {
-          // every earlier P V has to be done before O is touched
-          ok = __all_sync(0xffffffffu, mbar_wait(&pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1, p.status));
-          if (!ok) break;
-          tc_fence_after();
-#pragma unroll 1
-          for (int cc = 0; cc < D / 32; ++cc) {
-            uint32_t o[32];
-            tmem_ld32(tO + cc * 32 + lane_base, o);
-#pragma unroll
-            for (int k = 0; k < 32; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * factor);
-            tmem_st32(tO + cc * 32 + lane_base, o);
-          }
-        }
-        l *= factor;
-        const float nb = m == -INFINITY ? 0.f : -m;
-#pragma unroll 1
-        for (int ch = 0; ch < nch; ++ch) {
-          uint32_t sr[32];
-          tmem_ld32(tSb + ch * 32, sr);
-          const int kb = key0 + ch * 32;
-          const bool need_mask = kb + 31 > last_vis;
-          uint32_t pk[16];
-#pragma unroll
-          for (int c = 0; c < 32; c += 2) {
-            const float s0 = need_mask && kb + c > last_vis ? -INFINITY : __uint_as_float(sr[c]);
-            const float s1 = need_mask && kb + c + 1 > last_vis ? -INFINITY : __uint_as_float(sr[c + 1]);
-            const float p0 = fast_exp2(__fmaf_rn(s0, sl2, nb));
-            const float p1 = fast_exp2(__fmaf_rn(s1, sl2, nb));
-            l += p0 + p1;
-            pk[c >> 1] = pack_bf16x2(p0, p1);
-          }
-          tmem_st16(tSb + ch * 16, pk);
-        }
-      } else {
-        uint32_t pk[32];
-#pragma unroll
-        for (int c = 0; c < 32; ++c) pk[c] = 0u;
-#pragma unroll
-        for (int hh = 0; hh < kTcTile / 64; ++hh) tmem_st32(tSb + hh * 32, pk);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(q_ready);
       }
-      // V rows past kv_len may hold anything; zero them before P V reads them
-      if (key0 + kTcTile > U.kv_len) {
-        ok = __all_sync(0xffffffffu, mbar_wait(&v_full[st], (j / S) & 1, p.status));
+
+      const int last_vis = min(U.ctx + t, kv_end - 1);  // last key of this row in this split
+      // warps whose 32 rows are all padding write zero P, so every lane of P
+      // the tensor core reads is defined
+      const bool active = row0 + quad * 32 < M;
+      const float sl2 = p.scale_log2;
+      float m = -INFINITY, l = 0.f;
+      for (int j = 0; j < ntiles; ++j) {
+        const int gj = g0 + j;
+        const int b = gj & 1, st = gj % S;
+        const int key0 = kv_begin + j * kTcTile;
+        ok = __all_sync(0xffffffffu, mbar_wait(&s_full[b], (gj >> 1) & 1, p.status));
         if (!ok) break;
-        uint8_t* vt = sV + st * L::kTileBytes;
-        const int first = U.kv_len - key0;  // first key row to clear, up to the tile's loaded pages
-        const int nchunks = max(0, tile_pages(j) * kPage - first) * kHalves * 8;
-        for (int c = threadIdx.x - 64; c < nchunks; c += 128) {
-          const int row = first + c / (kHalves * 8);
-          const int rem = c % (kHalves * 8);  // every 16-byte chunk of the row, in any order
-          *reinterpret_cast<uint4*>(vt + (row / kPage) * L::kPageBytes + (rem >> 3) * (kPage * 128) +
-                                    (row % kPage) * 128 + ((rem & 7) << 4)) = make_uint4(0, 0, 0, 0);
+        tc_fence_after();
+        const uint32_t tSb = tS0 + b * kTcTile + lane_base;
+        if (active) {
+          // two passes over the tile's loaded columns in 32-column chunks (a
+          // small loop body: this code runs once per tile and per CTA, so its
+          // instruction fetch counts); the second pass overwrites S with P as it
+          // goes (P pairs of keys 32c..32c+31 land in columns 16c..16c+15, which
+          // this thread has already read)
+          const int nch = (tile_pages(j) * kPage + 31) / 32;
+          float mr = -INFINITY;
+#pragma unroll 1
+          for (int ch = 0; ch < nch; ++ch) {
+            uint32_t sr[32];
+            tmem_ld32(tSb + ch * 32, sr);
+            // raw scores; the causal rule key <= C_i + t only bites near the end
+            // (columns past the tile's pages are keys past kv_end: masked too)
+            const int kb = key0 + ch * 32;
+            const bool need_mask = kb + 31 > last_vis;
+#pragma unroll
+            for (int c = 0; c < 32; ++c) {
+              const float v = __uint_as_float(sr[c]);
+              mr = fmaxf(mr, need_mask && kb + c > last_vis ? -INFINITY : v);
+            }
+          }
+          const float mt = mr * sl2;  // tile maximum in log2 units (scale > 0)
+          // lazy rescale: keep the old maximum unless this tile exceeds it by 2^8
+          const bool grow = m == -INFINITY ? (mt > -INFINITY) : (mt > m + kRescaleThreshold);
+          float factor = 1.f;
+          if (grow) {
+            factor = m == -INFINITY ? 1.f : fast_exp2(m - mt);
+            m = mt;
+          }
+          if (j > 0 && __any_sync(0xffffffffu, grow && factor != 1.f)) {
+            // every earlier P V has to be done before O is touched
+            ok = __all_sync(0xffffffffu, mbar_wait(&pv_done[(gj - 1) & 1], ((gj - 1) >> 1) & 1, p.status));
+            if (!ok) break;
+            tc_fence_after();
+#pragma unroll 1
+            for (int cc = 0; cc < D / 32; ++cc) {
+              uint32_t o[32];
+              tmem_ld32(tO + cc * 32 + lane_base, o);
+#pragma unroll
+              for (int k = 0; k < 32; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * factor);
+              tmem_st32(tO + cc * 32 + lane_base, o);
+            }
+          }
+          l *= factor;
+          const float nb = m == -INFINITY ? 0.f : -m;
+#pragma unroll 1
+          for (int ch = 0; ch < nch; ++ch) {
+            uint32_t sr[32];
+            tmem_ld32(tSb + ch * 32, sr);
+            const int kb = key0 + ch * 32;
+            const bool need_mask = kb + 31 > last_vis;
+            uint32_t pk[16];
+#pragma unroll
+            for (int c = 0; c < 32; c += 2) {
+              const float s0 = need_mask && kb + c > last_vis ? -INFINITY : __uint_as_float(sr[c]);
+              const float s1 = need_mask && kb + c + 1 > last_vis ? -INFINITY : __uint_as_float(sr[c + 1]);
+              const float p0 = fast_exp2(__fmaf_rn(s0, sl2, nb));
+              const float p1 = fast_exp2(__fmaf_rn(s1, sl2, nb));
+              l += p0 + p1;
+              pk[c >> 1] = pack_bf16x2(p0, p1);
+            }
+            tmem_st16(tSb + ch * 16, pk);
+          }
+        } else {
+          uint32_t pk[32];
+#pragma unroll
+          for (int c = 0; c < 32; ++c) pk[c] = 0u;
+#pragma unroll
+          for (int hh = 0; hh < kTcTile / 64; ++hh) tmem_st32(tSb + hh * 32, pk);
         }
-        fence_proxy_async_smem();
+        // V rows past kv_len may hold anything; zero them before P V reads them
+        if (key0 + kTcTile > U.kv_len) {
+          ok = __all_sync(0xffffffffu, mbar_wait(&v_full[st], (gj / S) & 1, p.status));
+          if (!ok) break;
+          uint8_t* vt = sV + st * L::kTileBytes;
+          const int first = U.kv_len - key0;  // first key row to clear, up to the tile's loaded pages
+          const int nchunks = max(0, tile_pages(j) * kPage - first) * kHalves * 8;
+          for (int c = threadIdx.x - 64; c < nchunks; c += 128) {
+            const int row = first + c / (kHalves * 8);
+            const int rem = c % (kHalves * 8);  // every 16-byte chunk of the row, in any order
+            *reinterpret_cast<uint4*>(vt + (row / kPage) * L::kPageBytes + (rem >> 3) * (kPage * 128) +
+                                      (row % kPage) * 128 + ((rem & 7) << 4)) = make_uint4(0, 0, 0, 0);
+          }
+          fence_proxy_async_smem();
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&p_full[b]);
+      }
+
+      // ---- epilogue: O row from TMEM
+      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(o_final, n & 1, p.status));
+      fin_m = m;
+      fin_l = l;
+      fin_ok = ok;
+      if (ok && active && p.cluster <= 1) {
+        tc_fence_after();
+        const float inv = l > 0.f ? 1.f / l : 0.f;
+        __nv_bfloat16* orow = p.out + (static_cast<size_t>(U.q_off + t) * p.Hq + h * p.G + g) * D;
+        const long long prow_idx = p.part_off[ui] + static_cast<long long>(split * p.Hkv + h) * M + rg;
+#pragma unroll
+        for (int cc = 0; cc < D / 32; ++cc) {
+          uint32_t o[32];
+          tmem_ld32(tO + cc * 32 + lane_base, o);
+          if (!valid) continue;
+          if (U.nsplit == 1) {
+            uint4* dst = reinterpret_cast<uint4*>(orow + cc * 32);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              auto on = [&](int i) { return __uint_as_float(o[8 * k + i]) * inv; };
+              dst[k] = make_uint4(pack_bf16x2(on(0), on(1)), pack_bf16x2(on(2), on(3)), pack_bf16x2(on(4), on(5)),
+                                  pack_bf16x2(on(6), on(7)));
+            }
+          } else {
+            float4* dst = reinterpret_cast<float4*>(p.part_o + prow_idx * D + cc * 32);
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+              dst[k] = make_float4(__uint_as_float(o[4 * k]), __uint_as_float(o[4 * k + 1]),
+                                   __uint_as_float(o[4 * k + 2]), __uint_as_float(o[4 * k + 3]));
+          }
+        }
+        if (valid && U.nsplit > 1) p.part_ml[prow_idx] = make_float2(m, l);
       }
       tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&p_full[b]);
+      g0 += ntiles;
     }
-
-    // ---- epilogue: O row from TMEM
-    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(o_final, 0, p.status));
-    fin_m = m;
-    fin_l = l;
-    fin_ok = ok;
-    if (ok && active && p.cluster <= 1) {
-      tc_fence_after();
-      const float inv = l > 0.f ? 1.f / l : 0.f;
-      __nv_bfloat16* orow = p.out + (static_cast<size_t>(U.q_off + t) * p.Hq + h * p.G + g) * D;
-      const long long prow_idx = p.part_off[ui] + static_cast<long long>(split * p.Hkv + h) * M + rg;
-#pragma unroll
-      for (int cc = 0; cc < D / 32; ++cc) {
-        uint32_t o[32];
-        tmem_ld32(tO + cc * 32 + lane_base, o);
-        if (!valid) continue;
-        if (U.nsplit == 1) {
-          uint4* dst = reinterpret_cast<uint4*>(orow + cc * 32);
-#pragma unroll
-          for (int k = 0; k < 4; ++k)
-            dst[k] = make_uint4(pack_bf16x2(__uint_as_float(o[8 * k]) * inv, __uint_as_float(o[8 * k + 1]) * inv),
-                                pack_bf16x2(__uint_as_float(o[8 * k + 2]) * inv, __uint_as_float(o[8 * k + 3]) * inv),
-                                pack_bf16x2(__uint_as_float(o[8 * k + 4]) * inv, __uint_as_float(o[8 * k + 5]) * inv),
-                                pack_bf16x2(__uint_as_float(o[8 * k + 6]) * inv, __uint_as_float(o[8 * k + 7]) * inv));
-        } else {
-          float4* dst = reinterpret_cast<float4*>(p.part_o + prow_idx * D + cc * 32);
-#pragma unroll
-          for (int k = 0; k < 8; ++k)
-            dst[k] = make_float4(__uint_as_float(o[4 * k]), __uint_as_float(o[4 * k + 1]),
-                                 __uint_as_float(o[4 * k + 2]), __uint_as_float(o[4 * k + 3]));
-        }
-      }
-      if (valid && U.nsplit > 1) p.part_ml[prow_idx] = make_float2(m, l);
-    }
-    tc_fence_before();
   }
 
   if (p.cluster > 1) {

@@ -141,6 +141,7 @@ struct AttnPlan {
   int B = 0, Hq = 0, Hkv = 0, G = 0, D = 0;
   int NW = 4, stages = 3;
   int n_items = 0, n_merge = 0;
+  int grid = 0;     // CTAs launched: n_items, or fewer that each walk several items
   int cluster = 0;  // > 1: splits merged inside a thread-block cluster of this size
   long long part_rows = 0;
   std::vector<AttnUser> u;
@@ -176,7 +177,7 @@ int check_attn_users(int B, const int* L, const int* ctx, int Hq, int Hkv, int D
 static int split_pages(int pages, int ns) { return (pages + ns - 1) / ns; }
 
 void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int Hq, int Hkv, int D,
-                    int sms, AttnPlan& pl) {
+                    int sms, AttnPlan& pl, bool persist_ok = true) {
   pl.B = B; pl.Hq = Hq; pl.Hkv = Hkv; pl.G = Hq / Hkv; pl.D = D;
   int max_m = 0, max_tiles = 1;
   for (int i = 0; i < B; ++i) {
@@ -249,6 +250,60 @@ void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int
   }
   pl.cluster = (forced_cluster > 0 || best_b < best) && best_cl > 1 ? best_cl : 0;
 
+  // Persistent grid (more items than CTA slots): each CTA walks items
+  // blockIdx.x, + grid, ... and its K/V ring streams on across item
+  // boundaries, so an item costs its tiles plus ~0.5 (the softmax epilogue
+  // and the next Q) and a CTA ~2 once (prologue, last epilogue).  Cost: the
+  // most loaded CTA of that static assignment, items in launch order.  Not
+  // with the KV append (single-use patch barriers) nor the cluster merge.
+  int persist_mode = -1;  // -1: by cost, 0: never, 1: whenever allowed
+  int grid_cap = slots;
+  if (sms > 0) {  // forced for tests and tuning
+    if (const char* e = std::getenv("DIPSD_ATTN_PERSIST")) persist_mode = std::atoi(e) > 0 ? 1 : 0;
+    if (const char* e = std::getenv("DIPSD_ATTN_GRID")) grid_cap = std::max(1, std::min(slots, std::atoi(e)));
+  }
+  int best_pc = 0;
+  double best_p = 1e300;
+  if (persist_ok && pl.cluster <= 1 && persist_mode != 0) {
+    std::vector<double> load;
+    for (int c : cands) {
+      if (forced > 0) c = forced;
+      long long items = 0;
+      bool any_split = false;
+      for (int i = 0; i < B; ++i) {
+        const int tiles = (ctx[i] + L[i] + 1 + kTcTile - 1) / kTcTile;
+        const int pages = (ctx[i] + L[i] + 1 + kPage - 1) / kPage;
+        const int cc = std::max(1, std::min(c, tiles));
+        const int sp = split_pages(pages, (tiles + cc - 1) / cc);
+        const int ns = (pages + sp - 1) / sp;
+        items += static_cast<long long>(ns) * ((pl.G * (L[i] + 1) + rows_cta - 1) / rows_cta) * Hkv;
+        any_split = any_split || ns > 1;
+      }
+      const bool multi = items > grid_cap;
+      if ((multi || persist_mode > 0) && items <= 64ll * slots) {
+        const int grid = static_cast<int>(std::min<long long>(items, grid_cap));
+        load.assign(grid, 2.0);
+        long long it = 0;
+        for (int i = 0; i < B; ++i) {
+          const int tiles = (ctx[i] + L[i] + 1 + kTcTile - 1) / kTcTile;
+          const int pages = (ctx[i] + L[i] + 1 + kPage - 1) / kPage;
+          const int cc = std::max(1, std::min(c, tiles));
+          const int sp = split_pages(pages, (tiles + cc - 1) / cc);
+          const int ns = (pages + sp - 1) / sp;
+          const int reps = ((pl.G * (L[i] + 1) + rows_cta - 1) / rows_cta) * Hkv;  // (row block, head) pairs
+          for (int k = 0; k < reps; ++k)
+            for (int sidx = 0; sidx < ns; ++sidx, ++it)
+              load[it % grid] += std::min(sp, pages - sidx * sp) * kPage / 64.0 + 0.5;
+        }
+        const double cost = *std::max_element(load.begin(), load.end()) + (any_split ? 3.0 : 0.0);
+        if (cost < best_p - 1e-9) { best_p = cost; best_pc = c; }
+      }
+      if (forced > 0) break;
+    }
+  }
+  const bool persist = best_pc > 0 && (persist_mode > 0 || best_p < best);
+  if (persist) best_c = best_pc;
+
   pl.u.assign(B, AttnUser{});
   pl.item_off.assign(B + 1, 0);
   pl.merge_off.assign(B + 1, 0);
@@ -288,6 +343,7 @@ void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int
   pl.item_off[B] = static_cast<int>(items);
   pl.merge_off[B] = static_cast<int>(merge);
   pl.n_items = static_cast<int>(items);
+  pl.grid = persist ? std::min(pl.n_items, grid_cap) : pl.n_items;
   pl.n_merge = static_cast<int>(merge);
   pl.part_rows = part;
   pl.ws_bytes = part ? align_up(part * sizeof(float2), 256) + align_up(part * D * sizeof(float), 256) : 0;
@@ -320,14 +376,15 @@ void fill_attn_params(AttnParams<CAP>& p, const AttnPlan& pl, const void* q, voi
 template <int D, int CAP>
 int launch_attention_tc_t(const AttnPlan& pl, const AttnParams<CAP>& p, const CUtensorMap& tk,
                           const CUtensorMap& tv, cudaStream_t s, bool pdl) {
-  auto kern = verify_attention_tc_kernel<D, CAP>;
+  const bool persist = pl.grid < pl.n_items;
+  auto kern = persist ? verify_attention_tc_kernel<D, CAP, true> : verify_attention_tc_kernel<D, CAP, false>;
   static std::mutex mu;
-  static bool attr_done[64] = {};
+  static bool attr_done[2][64] = {};
   {
     std::lock_guard<std::mutex> lock(mu);
-    if (!allow_smem(kern, TcSmem<D>::kAlloc, attr_done)) return DIPSD_ERR_CUDA;
+    if (!allow_smem(kern, TcSmem<D>::kAlloc, attr_done[persist ? 1 : 0])) return DIPSD_ERR_CUDA;
   }
-  if (launch(kern, dim3(pl.n_items), dim3(kTcThreads), TcSmem<D>::kAlloc, s, pl.cluster > 1 ? pl.cluster : 0, pdl,
+  if (launch(kern, dim3(pl.grid), dim3(kTcThreads), TcSmem<D>::kAlloc, s, pl.cluster > 1 ? pl.cluster : 0, pdl,
              p, tk, tv) != cudaSuccess)
     return DIPSD_ERR_CUDA;
   if (pl.n_merge > 0) {
@@ -675,13 +732,20 @@ int dipsd_abi_version(void) { return DIPSD_ABI_VERSION; }
 
 long long dipsd_launch_count(void) { return g_launches; }
 
+// Attention workspace that covers the plans of both entry points (with and
+// without the KV append, which differ in their split choice).
+size_t attn_ws_need(int B, const int* L, const int* ctx, const int* bt_rows, int Hq, int Hkv, int D, int sms) {
+  AttnPlan a, b;
+  plan_attention(B, L, ctx, bt_rows, Hq, Hkv, D, sms, a, true);
+  plan_attention(B, L, ctx, bt_rows, Hq, Hkv, D, sms, b, false);
+  return std::max(a.ws_bytes, b.ws_bytes);
+}
+
 size_t dipsd_verify_attention_workspace_size(int B, const int* h_L, const int* h_ctx, int Hq, int Hkv, int D) {
   if (check_attn_users(B, h_L, h_ctx, Hq, Hkv, D) != DIPSD_OK) return 0;
   DeviceFacts f;
   if (!device_facts(f)) return 0;
-  AttnPlan pl;
-  plan_attention(B, h_L, h_ctx, nullptr, Hq, Hkv, D, f.sms, pl);
-  return kHeaderBytes + pl.ws_bytes;
+  return kHeaderBytes + attn_ws_need(B, h_L, h_ctx, nullptr, Hq, Hkv, D, f.sms);
 }
 
 static int verify_attention_impl(int B, const int* h_L, const int* h_ctx, const void* d_q, const void* d_k_cache,
@@ -696,7 +760,7 @@ static int verify_attention_impl(int B, const int* h_L, const int* h_ctx, const 
   DeviceFacts f;
   if (!device_facts(f)) return DIPSD_ERR_CUDA;
   AttnPlan pl;
-  plan_attention(B, h_L, h_ctx, nullptr, Hq, Hkv, D, f.sms, pl);
+  plan_attention(B, h_L, h_ctx, nullptr, Hq, Hkv, D, f.sms, pl, app.new_k == nullptr);
   st = check_workspace(d_workspace, workspace_bytes, kHeaderBytes + pl.ws_bytes);
   if (st != DIPSD_OK) return st;
   uint8_t* ws = static_cast<uint8_t*>(d_workspace);
@@ -856,9 +920,8 @@ size_t dipsd_verify_batch_workspace_size(int B, const int* h_members, int M, con
   if (check_spec_users(B, L.data(), V) != DIPSD_OK) return 0;
   DeviceFacts f;
   if (!device_facts(f)) return 0;
-  AttnPlan ap;
-  plan_attention(B, L.data(), ctx.data(), h_members, Hq, Hkv, D, f.sms, ap);
-  return kHeaderBytes + align_up(ap.ws_bytes, 256) + spec_ws_need(B, L.data(), V);
+  return kHeaderBytes + align_up(attn_ws_need(B, L.data(), ctx.data(), h_members, Hq, Hkv, D, f.sms), 256) +
+         spec_ws_need(B, L.data(), V);
 }
 
 static int verify_batch_impl(int B, const int* h_members, int M, const int* h_L_all, const int* h_ctx_all,
@@ -888,7 +951,7 @@ static int verify_batch_impl(int B, const int* h_members, int M, const int* h_L_
   DeviceFacts f;
   if (!device_facts(f)) return DIPSD_ERR_CUDA;
   AttnPlan ap;
-  plan_attention(B, L.data(), ctx.data(), h_members, Hq, Hkv, D, f.sms, ap);
+  plan_attention(B, L.data(), ctx.data(), h_members, Hq, Hkv, D, f.sms, ap, app.new_k == nullptr);
   SpecPlan sp;
   plan_spec(B, L.data(), V, logit_dtype == DIPSD_BF16 ? 2 : 4, vec_ok, f.sms, sp);
   const size_t attn_region = align_up(ap.ws_bytes, 256);

@@ -73,7 +73,8 @@ def test_append_attention_edges(cuda_lib, L, ctx, Hq, Hkv, D):
 
 
 @pytest.mark.parametrize("env,val", [("DIPSD_ATTN_SPLIT_TILES", "1"), ("DIPSD_ATTN_SPLIT_TILES", "3"),
-                                     ("DIPSD_ATTN_CLUSTER", "3")])
+                                     ("DIPSD_ATTN_CLUSTER", "3"),
+                                     ("DIPSD_ATTN_PERSIST", "1")])
 def test_append_with_splits(cuda_lib, env, val):
     """Splits of one tile each put the new rows of a user into two CTAs."""
     b = make_batch([31, 5, 0, 12], [50, 1000, 63, 200], Hq=64, Hkv=8, D=128, V=64, seed=47)

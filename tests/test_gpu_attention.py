@@ -94,6 +94,33 @@ def test_attention_cluster_merge(cuda_lib, cluster, D):
     check_attention(out, _full_reference(b))
 
 
+@pytest.mark.parametrize("grid,split_tiles,D", [("1", None, 128), ("3", None, 128), ("7", "2", 128),
+                                                 ("5", "1", 64), ("152", "1", 128)])
+def test_attention_persistent_grid(cuda_lib, grid, split_tiles, D):
+    """A grid smaller than the item count: each CTA walks several items (row
+    blocks with and without padding rows, ragged last tiles, KV splits and
+    their merge), the K/V ring and every barrier phase running on across
+    items."""
+    b = make_batch([5, 0, 8, 2, 20, 1], [1500, 3000, 333, 64, 700, 0], Hq=64 if D == 128 else 16,
+                   Hkv=8 if D == 128 else 2, D=D, V=64, seed=24)
+    env = {"DIPSD_ATTN_PERSIST": "1", "DIPSD_ATTN_GRID": grid}
+    if split_tiles:
+        env["DIPSD_ATTN_SPLIT_TILES"] = split_tiles
+    old = {k: os.environ.get(k) for k in env}
+    os.environ.update(env)
+    try:
+        ws = cuda_lib.workspace(cuda_lib.dipsd_verify_attention_workspace_size(b.L, b.ctx, b.Hq, b.Hkv, b.D), DEV)
+        out = _run(cuda_lib, b, ws)
+        assert cuda_lib.device_status(ws) == 0
+    finally:
+        for k, v in old.items():
+            if v is None:
+                del os.environ[k]
+            else:
+                os.environ[k] = v
+    check_attention(out, _full_reference(b))
+
+
 def test_attention_ignores_slots_past_kv_len(cuda_lib):
     """NaN in cache slots past each user's kv_len and in unused pages never reaches the output."""
     b = make_batch([2, 5, 0], [30, 500, 1], Hq=64, Hkv=8, D=128, V=64, seed=22)
