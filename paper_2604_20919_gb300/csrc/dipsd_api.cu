@@ -770,6 +770,25 @@ static int verify_attention_impl(int B, const int* h_L, const int* h_ctx, const 
   return st != DIPSD_OK ? st : cuda_status();
 }
 
+int dipsd_verify_attention_plan(int B, const int* h_L, const int* h_ctx, int Hq, int Hkv, int D, int num_sms,
+                                int append, dipsd_attention_plan* out, int* h_nsplit, int* h_split_len) {
+  const int st = check_attn_users(B, h_L, h_ctx, Hq, Hkv, D);
+  if (st != DIPSD_OK) return st;
+  if (num_sms < 1 || !out) return DIPSD_ERR_INVALID_ARG;
+  AttnPlan pl;
+  plan_attention(B, h_L, h_ctx, nullptr, Hq, Hkv, D, num_sms, pl, append == 0);
+  out->n_items = pl.n_items;
+  out->grid = pl.grid;
+  out->cluster = pl.cluster > 1 ? pl.cluster : 0;
+  out->n_merge = pl.n_merge;
+  out->ws_bytes = pl.ws_bytes;
+  for (int i = 0; i < B; ++i) {
+    if (h_nsplit) h_nsplit[i] = pl.u[i].nsplit;
+    if (h_split_len) h_split_len[i] = pl.u[i].split_len;
+  }
+  return DIPSD_OK;
+}
+
 int dipsd_verify_attention(int B, const int* h_L, const int* h_ctx, const void* d_q, const void* d_k_cache,
                            const void* d_v_cache, int num_blocks, const int* d_block_table, int max_blocks,
                            int Hq, int Hkv, int D, float softmax_scale, void* d_out, void* d_workspace,

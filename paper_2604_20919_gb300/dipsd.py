@@ -34,7 +34,7 @@ EXPORTS = (
     "dipsd_spec_verify_workspace_size", "dipsd_spec_verify",
     "dipsd_verify_batch_workspace_size", "dipsd_verify_batch", "dipsd_spec_verify_noalloc",
     "dipsd_verify_attention_append", "dipsd_verify_batch_append",
-    "dipsd_spec_verify_sparse_workspace_size", "dipsd_spec_verify_sparse",
+    "dipsd_spec_verify_sparse_workspace_size", "dipsd_spec_verify_sparse", "dipsd_verify_attention_plan",
 )
 NOALLOC_MAX_POSITIONS = 4096
 
@@ -43,6 +43,11 @@ _i32p = ctypes.POINTER(ctypes.c_int)
 _vp = ctypes.c_void_p
 _sz = ctypes.c_size_t
 _i = ctypes.c_int
+
+
+class AttentionPlan(ctypes.Structure):
+    """dipsd_attention_plan of include/dipsd.h."""
+    _fields_ = [("n_items", _i), ("grid", _i), ("cluster", _i), ("n_merge", _i), ("ws_bytes", _sz)]
 
 
 class DipsdError(RuntimeError):
@@ -90,6 +95,9 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.dipsd_spec_verify_sparse.restype = _i
     lib.dipsd_spec_verify_sparse.argtypes = [_i, _i32p, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
                                              _vp, _sz, _vp]
+    lib.dipsd_verify_attention_plan.restype = _i
+    lib.dipsd_verify_attention_plan.argtypes = [_i, _i32p, _i32p, _i, _i, _i, _i, _i,
+                                                ctypes.POINTER(AttentionPlan), _i32p, _i32p]
     lib.dipsd_spec_verify_noalloc.restype = _i
     lib.dipsd_spec_verify_noalloc.argtypes = [_i, _i32p, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]
     _lib = lib
@@ -156,6 +164,21 @@ def dipsd_verify_attention_workspace_size(L, ctx, Hq: int, Hkv: int, D: int) -> 
     a, pa = _host_i32(L)
     b, pb = _host_i32(ctx)
     return int(load().dipsd_verify_attention_workspace_size(len(a), pa, pb, Hq, Hkv, D))
+
+
+def dipsd_verify_attention_plan(L, ctx, Hq: int, Hkv: int, D: int, num_sms: int, append: bool = False) -> dict:
+    """The work-item plan the attention entry points make for a device with
+    num_sms SMs (host only).  Returns n_items, grid, cluster, n_merge,
+    ws_bytes and per user nsplit and split_len."""
+    a, pa = _host_i32(L)
+    b, pb = _host_i32(ctx)
+    plan = AttentionPlan()
+    nsplit, pn = _host_i32(np.zeros(len(a)))
+    split_len, ps = _host_i32(np.zeros(len(a)))
+    _check(load().dipsd_verify_attention_plan(len(a), pa, pb, Hq, Hkv, D, int(num_sms), 1 if append else 0,
+                                              ctypes.byref(plan), pn, ps), "dipsd_verify_attention_plan")
+    return {"n_items": plan.n_items, "grid": plan.grid, "cluster": plan.cluster, "n_merge": plan.n_merge,
+            "ws_bytes": int(plan.ws_bytes), "nsplit": nsplit, "split_len": split_len}
 
 
 def dipsd_verify_attention(L, ctx, q, k_cache, v_cache, block_table, softmax_scale: float, out=None,
