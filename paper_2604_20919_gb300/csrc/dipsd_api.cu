@@ -265,10 +265,20 @@ void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int
   int best_pc = 0;
   double best_p = 1e300;
   if (persist_ok && pl.cluster <= 1 && persist_mode != 0) {
-    std::vector<double> load;
+    // Per candidate: the split of every user, the item count and a lower
+    // bound on the most loaded CTA (the mean load); the exact static
+    // assignment is then costed in ascending bound order until the bound
+    // passes the best cost found (same choice as costing every candidate).
+    struct Cand {
+      int c, grid;
+      bool any_split;
+      double bound;
+    };
+    std::vector<Cand> cs;
     for (int c : cands) {
       if (forced > 0) c = forced;
       long long items = 0;
+      double total = 0;
       bool any_split = false;
       for (int i = 0; i < B; ++i) {
         const int tiles = (ctx[i] + L[i] + 1 + kTcTile - 1) / kTcTile;
@@ -276,29 +286,49 @@ void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int
         const int cc = std::max(1, std::min(c, tiles));
         const int sp = split_pages(pages, (tiles + cc - 1) / cc);
         const int ns = (pages + sp - 1) / sp;
-        items += static_cast<long long>(ns) * ((pl.G * (L[i] + 1) + rows_cta - 1) / rows_cta) * Hkv;
+        const long long reps = static_cast<long long>((pl.G * (L[i] + 1) + rows_cta - 1) / rows_cta) * Hkv;
+        items += ns * reps;
+        total += reps * (pages * kPage / 64.0 + 0.5 * ns);
         any_split = any_split || ns > 1;
       }
-      const bool multi = items > grid_cap;
-      if ((multi || persist_mode > 0) && items <= 64ll * slots) {
+      if ((items > grid_cap || persist_mode > 0) && items <= 64ll * slots) {
         const int grid = static_cast<int>(std::min<long long>(items, grid_cap));
-        load.assign(grid, 2.0);
-        long long it = 0;
-        for (int i = 0; i < B; ++i) {
-          const int tiles = (ctx[i] + L[i] + 1 + kTcTile - 1) / kTcTile;
-          const int pages = (ctx[i] + L[i] + 1 + kPage - 1) / kPage;
-          const int cc = std::max(1, std::min(c, tiles));
-          const int sp = split_pages(pages, (tiles + cc - 1) / cc);
-          const int ns = (pages + sp - 1) / sp;
-          const int reps = ((pl.G * (L[i] + 1) + rows_cta - 1) / rows_cta) * Hkv;  // (row block, head) pairs
-          for (int k = 0; k < reps; ++k)
-            for (int sidx = 0; sidx < ns; ++sidx, ++it)
-              load[it % grid] += std::min(sp, pages - sidx * sp) * kPage / 64.0 + 0.5;
-        }
-        const double cost = *std::max_element(load.begin(), load.end()) + (any_split ? 3.0 : 0.0);
-        if (cost < best_p - 1e-9) { best_p = cost; best_pc = c; }
+        cs.push_back({c, grid, any_split, 2.0 + total / grid + (any_split ? 3.0 : 0.0)});
       }
       if (forced > 0) break;
+    }
+    std::stable_sort(cs.begin(), cs.end(), [](const Cand& x, const Cand& y) { return x.bound < y.bound; });
+    std::vector<double> load;
+    int best_rank = 1 << 30;  // position in `cands` of the best candidate (ties: the first, as listed)
+    auto rank_of = [&](int c) {
+      return static_cast<int>(std::find(std::begin(cands), std::end(cands), c) - std::begin(cands));
+    };
+    for (const Cand& k : cs) {
+      if (k.bound > best_p + 1e-9) break;
+      load.assign(k.grid, 2.0);
+      int slot = 0;  // CTA of the next item: items go round-robin over the grid
+      for (int i = 0; i < B; ++i) {
+        const int tiles = (ctx[i] + L[i] + 1 + kTcTile - 1) / kTcTile;
+        const int pages = (ctx[i] + L[i] + 1 + kPage - 1) / kPage;
+        const int cc = std::max(1, std::min(k.c, tiles));
+        const int sp = split_pages(pages, (tiles + cc - 1) / cc);
+        const int ns = (pages + sp - 1) / sp;
+        const int reps = ((pl.G * (L[i] + 1) + rows_cta - 1) / rows_cta) * Hkv;  // (row block, head) pairs
+        const double full = sp * kPage / 64.0 + 0.5;                           // every split but the last
+        const double last = (pages - (ns - 1) * sp) * kPage / 64.0 + 0.5;
+        for (int r = 0; r < reps; ++r)
+          for (int sidx = 0; sidx < ns; ++sidx) {
+            load[slot] += sidx + 1 < ns ? full : last;
+            if (++slot == k.grid) slot = 0;
+          }
+      }
+      const double cost = *std::max_element(load.begin(), load.end()) + (k.any_split ? 3.0 : 0.0);
+      const int rank = rank_of(k.c);
+      if (cost < best_p - 1e-9 || (cost <= best_p + 1e-9 && rank < best_rank)) {
+        best_p = cost;
+        best_pc = k.c;
+        best_rank = rank;
+      }
     }
   }
   const bool persist = best_pc > 0 && (persist_mode > 0 || best_p < best);
