@@ -84,7 +84,6 @@ struct TcSmem {
 static_assert((TcSmem<128>::kMaxCluster - 1) * TcSmem<128>::kSlotBytes <= TcSmem<128>::kVOff, "exchange fits");
 static_assert((TcSmem<64>::kMaxCluster - 1) * TcSmem<64>::kSlotBytes <= TcSmem<64>::kVOff, "exchange fits");
 static_assert(TcSmem<128>::kAlloc <= 232448 && TcSmem<64>::kAlloc <= 232448, "shared memory per CTA");
-constexpr int kTcStages = TcSmem<128>::kStages;
 
 // tm_k: 4-D {64 columns, 16 rows, heads, blocks}, one 64-column half of a
 // page per box; tm_v: 5-D {64 columns, 16 rows, halves, heads, blocks}, a

@@ -139,7 +139,6 @@ bool allow_smem(K kernel, int bytes, bool* done) {
 // =================================================================== attention
 struct AttnPlan {
   int B = 0, Hq = 0, Hkv = 0, G = 0, D = 0;
-  int NW = 4, stages = 3;
   int n_items = 0, n_merge = 0;
   int grid = 0;     // CTAs launched: n_items, or fewer that each walk several items
   int cluster = 0;  // > 1: splits merged inside a thread-block cluster of this size
@@ -147,7 +146,6 @@ struct AttnPlan {
   std::vector<AttnUser> u;
   std::vector<int> item_off, merge_off;
   std::vector<long long> part_off;
-  size_t smem = 0;
   size_t ws_bytes = 0;  // attention region only (excludes the status word)
 };
 
@@ -179,15 +177,8 @@ static int split_pages(int pages, int ns) { return (pages + ns - 1) / ns; }
 void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int Hq, int Hkv, int D,
                     int sms, AttnPlan& pl, bool persist_ok = true) {
   pl.B = B; pl.Hq = Hq; pl.Hkv = Hkv; pl.G = Hq / Hkv; pl.D = D;
-  int max_m = 0, max_tiles = 1;
-  for (int i = 0; i < B; ++i) {
-    max_m = std::max(max_m, pl.G * (L[i] + 1));
-    max_tiles = std::max(max_tiles, (ctx[i] + L[i] + 1 + kTcTile - 1) / kTcTile);
-  }
-  // tcgen05 kernel: 128 rows per CTA, one CTA per SM (its shared memory)
-  pl.NW = 8;
-  pl.stages = kTcStages;
-  pl.smem = D == 128 ? TcSmem<128>::kAlloc : TcSmem<64>::kAlloc;
+  // tcgen05 kernel: 128 rows per CTA, one CTA per SM (its shared memory and
+  // all of tensor memory)
   const int rows_cta = 128;
   const int slots = sms;
 
