@@ -1,9 +1,13 @@
 // verify_attention on the 5th-generation tensor cores (tcgen05 + TMEM).
 //
-// Work decomposition: one CTA per (user i, KV head h, row block, KV split);
-// rows r = t*G + g pack the G query heads of the KV group and the T_i verify
-// tokens (Sec. II-A stage 2: all L_i+1 tokens of a user are verified in one
-// pass), so each K/V byte brought on chip serves every row.
+// Work decomposition: a work item is (user i, KV head h, row block, KV
+// split); rows r = t*G + g pack the G query heads of the KV group and the T_i
+// verify tokens (Sec. II-A stage 2: all L_i+1 tokens of a user are verified
+// in one pass), so each K/V byte brought on chip serves every row.  One CTA
+// per item, or (PERSIST) a grid of at most one CTA per SM in which CTA b
+// takes items b, b + gridDim.x, ...: the rings, the S/P buffers and every
+// barrier phase then run on across items, so the producer streams the next
+// item's tiles while the softmax warps finish the current one.
 //
 // Roles (6 warps):
 //   warp 0      TMA producer into a ring of kStages 128-token K tiles and
