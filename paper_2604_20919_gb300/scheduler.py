@@ -454,3 +454,48 @@ def fixed_lengths(p: SystemParams, l: int = 7) -> Plan:
         if best is None or plan.throughput > best.throughput:
             best = plan
     return best
+
+
+# ----------------------------------------------------------------- command line
+def main(argv: Optional[Sequence[str]] = None) -> dict:
+    """Plans M users under Table 2's defaults (per-user acceptance rates and
+    prefix lengths may be given) and prints one JSON line: the plan, its
+    throughput and the Sec. IV-A baselines, all in tokens per second."""
+    import argparse
+    import json
+    ap = argparse.ArgumentParser(prog="python -m paper_2604_20919_gb300.scheduler",
+                                 description="DiP-SD batch planning (Algorithm 1) under the paper's latency model")
+    ap.add_argument("--users", type=int, default=6, help="M")
+    ap.add_argument("--alpha", type=float, nargs="+", default=[0.78], help="one acceptance rate, or one per user")
+    ap.add_argument("--prefix", type=int, nargs="+", default=[512], help="one prefix length, or one per user")
+    ap.add_argument("--l-max", type=int, default=20, help="L_ub")
+    ap.add_argument("--mem-cap", type=float, default=8.0e10, help="Gamma_max in bytes")
+    args = ap.parse_args(argv)
+    M = args.users
+    if M < 2:
+        ap.error("--users must be at least 2 (the plan has N >= 2 batches)")
+
+    def per_user(v, name):
+        if len(v) == 1:
+            return list(v) * M
+        if len(v) != M:
+            ap.error(f"--{name} takes 1 or {M} values")
+        return list(v)
+
+    p = SystemParams.homogeneous(M, l_max=args.l_max, mem_cap=args.mem_cap)
+    p.alpha = per_user(args.alpha, "alpha")
+    p.prefix = per_user(args.prefix, "prefix")
+    plan = solve(p)
+    out = {"throughput_tokens_per_s": 1000.0 * plan.throughput, "N": plan.N, "batches": plan.batches,
+           "draft_len": plan.draft_len, "U": plan.U, "S_ms": plan.S,
+           "baselines_tokens_per_s": {
+               "AD": 1000.0 * autoregressive(p),
+               "AD_greedy_batching": 1000.0 * autoregressive_greedy(p),
+               "without_batching": 1000.0 * without_batching(p).throughput,
+               "fixed_l7": 1000.0 * fixed_lengths(p, min(7, p.l_max)).throughput}}
+    print(json.dumps(out))
+    return out
+
+
+if __name__ == "__main__":
+    main()

@@ -82,3 +82,23 @@ def test_greedy_batching_packs_by_prefix():
     J, h1 = p.verify.J, p.verify.h1
     p.mem_cap = sc.param_bytes(p) + 4.0 * J * h1 * 2 * 800 + 1.0
     assert sc.greedy_batches(p) == [[1, 3], [2, 0]]
+
+
+def test_command_line_plan(capsys):
+    """`python -m paper_2604_20919_gb300.scheduler` prints the plan and the
+    baselines; at M = 6, alpha = 0.95 they are the paper's printed figures."""
+    out = sc.main(["--users", "6", "--alpha", "0.95"])
+    printed = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert printed["N"] == out["N"] and printed["batches"] == out["batches"]
+    gold = GOLD["alpha_sweep_M6"]
+    assert round(out["throughput_tokens_per_s"], 2) == gold["dipsd_alpha_0.95"]
+    base = out["baselines_tokens_per_s"]
+    assert round(out["throughput_tokens_per_s"] / base["AD"], 2) == gold["speedup_vs_ad_alpha_0.95"]
+    assert round(out["throughput_tokens_per_s"] / base["AD_greedy_batching"], 2) == \
+        gold["speedup_vs_ad_greedy_alpha_0.95"]
+    assert sorted(m for b in out["batches"] for m in b) == list(range(6))
+    # per-user values: one per user, or the run stops with a usage error
+    out = sc.main(["--users", "3", "--alpha", "0.7", "0.8", "0.9", "--prefix", "300", "500", "700"])
+    assert sorted(m for b in out["batches"] for m in b) == [0, 1, 2]
+    with pytest.raises(SystemExit):
+        sc.main(["--users", "3", "--alpha", "0.7", "0.8"])
