@@ -77,7 +77,8 @@ def _enumerated_law(zl, wl, L):
     V = zl.shape[1]
     p = scipy.special.softmax(zl, axis=-1)
     q = scipy.special.softmax(wl, axis=-1) if L else np.zeros((0, V))
-    acc_cells = [_cells(np.minimum(1.0, p[t] / q[t])) for t in range(L)]
+    with np.errstate(divide="ignore"):  # q(d) = 0: the ratio is +inf and min(1, .) = 1
+        acc_cells = [_cells(np.minimum(1.0, p[t] / q[t])) for t in range(L)]
     res_cells = []
     for t in range(L + 1):
         pts = [np.cumsum(p[t])]
