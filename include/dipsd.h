@@ -21,7 +21,9 @@
  *                           K/V rows into their pages in the same launch;
  *   dipsd_spec_verify_sparse  speculative sampling from a sparse draft
  *                           payload (draft-token log-probabilities and a
- *                           top-K draft distribution).
+ *                           top-K draft distribution);
+ *   dipsd_verify_attention_plan  the attention's work-item plan for a given
+ *                           SM count (host only).
  *
  * Conventions shared by every entry point
  *   - Pointers named d_* are device pointers, h_* host pointers.  The caller
