@@ -1,7 +1,6 @@
 """verify_attention through the C ABI vs the fp64 oracle."""
 import os
 
-import numpy as np
 import pytest
 import torch
 

@@ -6,7 +6,7 @@ import pytest
 import scipy.stats
 import torch
 
-from parity import check_spec, spec_reference, valid_spec_outputs
+from parity import check_spec, valid_spec_outputs
 from workloads import make_batch, make_config
 
 pytestmark = pytest.mark.gpu
