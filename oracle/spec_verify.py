@@ -34,7 +34,9 @@ Pins (tests/test_oracle_spec.py): scipy softmax; exact brute force of the
 whole output law on tiny vocabularies against the closed form
 prod_t min(p_t, q_t) * (residual or p); Monte Carlo chi-square of the
 emitted tokens against p; acceptance rate sum_v min(p, q); expected length
-(1 - alpha^(L+1)) / (1 - alpha), Eq. (u_single).
+(1 - alpha^(L+1)) / (1 - alpha), Eq. (u_single).  The boundary-band helpers
+(_cdf_margin, margin_accept, decision_margins) are pinned on hand-worked
+values in tests/test_oracle_margins.py.
 """
 from __future__ import annotations
 
