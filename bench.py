@@ -254,7 +254,7 @@ def run_dipsd(args):
         kc = b.k_cache if k == 0 else b.k_cache.clone()
         vc = b.v_cache if k == 0 else b.v_cache.clone()
         copies.append(dict(q=b.q.to(dev), z=b.target_logits.to(dev), w=b.draft_logits.to(dev),
-                           d=b.draft_tokens.to(dev), u=b.uniforms.to(dev), kc=kc, vc=vc))
+                           d=b.draft_tokens.to(dev), kc=kc, vc=vc))
     bt = b.block_table.to(dev)
     attn_out = torch.empty_like(copies[0]["q"])
     outs = dipsd.spec_outputs(b.L, dev)
@@ -265,7 +265,7 @@ def run_dipsd(args):
     def step(k):
         c = copies[k % R]
         dipsd.dipsd_verify_batch(b.members, b.L, b.ctx, c["q"], c["kc"], c["vc"], bt, b.scale, c["z"], c["w"],
-                                 c["d"], c["u"], attn_out=attn_out, outputs=outs, ws=ws)
+                                 c["d"], b.seed, attn_out=attn_out, outputs=outs, ws=ws)
 
     def attn_only(k):
         c = copies[k % R]
@@ -273,7 +273,7 @@ def run_dipsd(args):
 
     def spec_only(k):
         c = copies[k % R]
-        dipsd.dipsd_spec_verify(b.L, c["z"], c["w"], c["d"], c["u"], outputs=outs, ws=ws)
+        dipsd.dipsd_spec_verify(b.L, b.members, b.seed, c["z"], c["w"], c["d"], outputs=outs, ws=ws)
 
     # the verify tokens' own K/V rows (already in the cache), for the append path
     bt_h = b.block_table.numpy()
@@ -292,8 +292,8 @@ def run_dipsd(args):
 
     def spec_sparse(k):
         c = copies[k % R]
-        dipsd.dipsd_spec_verify_sparse(b.L, c["z"], sd_dev["draft_tokens"], sd_dev["draft_logq"], sd_dev["topk_idx"],
-                                       sd_dev["topk_q"], c["u"], outputs=sp_outs, ws=ws_sp)
+        dipsd.dipsd_spec_verify_sparse(b.L, b.members, b.seed, c["z"], sd_dev["draft_tokens"], sd_dev["draft_logq"],
+                                       sd_dev["topk_idx"], sd_dev["topk_q"], outputs=sp_outs, ws=ws_sp)
 
     def attn_append(k):
         c = copies[k % R]
@@ -374,8 +374,8 @@ def run_dipsd(args):
     # step k+1's upload overlaps step k's compute.  R steps are captured as one
     # graph, replayed back to back, timed on the host clock.
     pin = lambda t: t.cpu().pin_memory()
-    keys = ("q", "z", "w", "d", "u")
-    h_in = [pin(x) for x in (b.q, b.target_logits, b.draft_logits, b.draft_tokens, b.uniforms)]
+    keys = ("q", "z", "w", "d")
+    h_in = [pin(x) for x in (b.q, b.target_logits, b.draft_logits, b.draft_tokens)]
     h_out = [[torch.empty_like(x, device="cpu").pin_memory() for x in outs[:3]] for _ in range(R)]
     h2d = sum(x.numel() * x.element_size() for x in h_in)
     d2h = sum(x.numel() * x.element_size() for x in h_out[0])
@@ -474,7 +474,7 @@ def run_dipsd(args):
         "step_latency_cold_l2_ms": lat_step,
         "e2e": {"value": units_all / (e2e_max / 1000.0), "unit": "verified tokens/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                "schedule": "per step: pinned H2D of q, logits, drafts, uniforms; the call; D2H of "
+                "schedule": "per step: pinned H2D of q, logits, drafts; the call; D2H of "
                             "accept_len, offsets, tokens; uploads overlap the previous step's compute",
                 "ms_per_step": e2e_max / args.steps},
         "gpu_launches": int(launches),
@@ -514,7 +514,7 @@ def run_pipeline(args):
         ws = dipsd.workspace(dipsd.dipsd_verify_batch_workspace_size(b.members, L_all, ctx_all, b.Hq, b.Hkv, b.D,
                                                                      b.V), dev)
         stage.append(dict(b=b, q=g(b.q), z=g(b.target_logits), w=g(b.draft_logits), d=g(b.draft_tokens),
-                          u=g(b.uniforms), attn=torch.empty_like(b.q, device=dev),
+                          attn=torch.empty_like(b.q, device=dev),
                           outs=dipsd.spec_outputs(b.L, dev), ws=ws, stream=streams[n % 2]))
     main = torch.cuda.current_stream()
 
@@ -526,7 +526,8 @@ def run_pipeline(args):
             for x in stage:
                 with torch.cuda.stream(x["stream"]):
                     dipsd.dipsd_verify_batch(x["b"].members, L_all, ctx_all, x["q"], kc, vc, bt, x["b"].scale,
-                                             x["z"], x["w"], x["d"], x["u"], attn_out=x["attn"], outputs=x["outs"],
+                                             x["z"], x["w"], x["d"], x["b"].seed, attn_out=x["attn"],
+                                             outputs=x["outs"],
                                              ws=x["ws"], stream=x["stream"])
         for sm in streams:
             cur.wait_stream(sm)

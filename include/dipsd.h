@@ -23,7 +23,10 @@
  *                           payload (draft-token log-probabilities and a
  *                           top-K draft distribution);
  *   dipsd_verify_attention_plan  the attention's work-item plan for a given
- *                           SM count (host only).
+ *                           SM count (host only);
+ *   dipsd_philox_words,
+ *   dipsd_verify_uniforms   the random numbers speculative sampling draws
+ *                           (in-kernel Philox4x64-10), written out.
  *
  * Conventions shared by every entry point
  *   - Pointers named d_* are device pointers, h_* host pointers.  The caller
@@ -56,7 +59,7 @@
 extern "C" {
 #endif
 
-#define DIPSD_ABI_VERSION 1
+#define DIPSD_ABI_VERSION 2
 #define DIPSD_PAGE_SIZE 16    /* tokens per KV page */
 #define DIPSD_MAX_USERS 512   /* users per call */
 #define DIPSD_MAX_DRAFT 31    /* L_i <= 31: one warp ballot covers a user */
@@ -166,14 +169,22 @@ int dipsd_verify_attention_plan(int B, const int* h_L, const int* h_ctx, int Hq,
  *   max(0, p_a - q_a)  if a_i < L_i (p_a itself if that has no mass),
  *   p_{L_i}            if a_i == L_i (the bonus position).
  *
+ * The uniforms are drawn inside the kernels (the paper leaves them
+ * unspecified): user i's stream is Philox4x64-10 (Salmon et al., SC 2011)
+ * under the 128-bit key (seed, h_user_id[i]), counter blocks (1,0,0,0),
+ * (2,0,0,0), ...; verify position t takes the stream's 64-bit words 2t
+ * (u_acc) and 2t+1 (u_res), each mapped to ((w >> 41) + 0.5) * 2^-23, an
+ * exact fp32 in (0, 1).  The same (seed, user id) always gives the same
+ * uniforms; dipsd_verify_uniforms writes them out.
+ *
  * B                  1..DIPSD_MAX_USERS;  h_L [B] host, 0..DIPSD_MAX_DRAFT
+ * h_user_id          [B] host, >= 0: Philox key word 1 of each user
+ * seed               Philox key word 0
  * V                  vocabulary size >= 1
  * logit_dtype        DIPSD_BF16 or DIPSD_F32 (both logit arrays)
  * d_target_logits    [sum_i (L_i+1)][V], user i's rows in position order
  * d_draft_logits     [sum_i L_i][V]
  * d_draft_tokens     [sum_i L_i] int32 in [0, V)
- * d_uniforms         [sum_i (L_i+1)][2] fp32 in (0,1): (u_acc, u_res) per
- *                    verify position (u_acc of the bonus position is unused)
  * d_accept_len       [B] int32 out: a_i
  * d_out_offsets      [B+1] int32 out: exclusive prefix of (a_i + 1)
  * d_out_tokens       [sum_i (L_i+1)] int32 out (capacity); the first
@@ -183,12 +194,11 @@ int dipsd_verify_attention_plan(int B, const int* h_L, const int* h_ctx, int Hq,
  * Rows must start 16-byte aligned for the fast path (V*elem % 16 == 0).
  * ---------------------------------------------------------------------- */
 size_t dipsd_spec_verify_workspace_size(int B, const int* h_L, int V);
-int dipsd_spec_verify(int B, const int* h_L, int V, int logit_dtype,
-                      const void* d_target_logits, const void* d_draft_logits,
-                      const int* d_draft_tokens, const float* d_uniforms,
-                      int* d_accept_len, int* d_out_offsets, int* d_out_tokens,
-                      float* d_draft_probs, void* d_workspace, size_t workspace_bytes,
-                      void* stream);
+int dipsd_spec_verify(int B, const int* h_L, const int* h_user_id, uint64_t seed, int V,
+                      int logit_dtype, const void* d_target_logits, const void* d_draft_logits,
+                      const int* d_draft_tokens, int* d_accept_len, int* d_out_offsets,
+                      int* d_out_tokens, float* d_draft_probs, void* d_workspace,
+                      size_t workspace_bytes, void* stream);
 
 /* ------------------------------------------------------------------------
  * Speculative verification from a sparse draft payload (Sec. II-A: the device
@@ -210,13 +220,12 @@ int dipsd_spec_verify(int B, const int* h_L, int V, int logit_dtype,
  * (p_t(d), exp(draft_logq)).
  * ---------------------------------------------------------------------- */
 size_t dipsd_spec_verify_sparse_workspace_size(int B, const int* h_L, int V);
-int dipsd_spec_verify_sparse(int B, const int* h_L, int V, int K, int logit_dtype,
-                             const void* d_target_logits, const int* d_draft_tokens,
-                             const float* d_draft_logq, const int* d_topk_idx,
-                             const float* d_topk_q, const float* d_uniforms,
-                             int* d_accept_len, int* d_out_offsets, int* d_out_tokens,
-                             float* d_draft_probs, void* d_workspace, size_t workspace_bytes,
-                             void* stream);
+int dipsd_spec_verify_sparse(int B, const int* h_L, const int* h_user_id, uint64_t seed, int V,
+                             int K, int logit_dtype, const void* d_target_logits,
+                             const int* d_draft_tokens, const float* d_draft_logq,
+                             const int* d_topk_idx, const float* d_topk_q, int* d_accept_len,
+                             int* d_out_offsets, int* d_out_tokens, float* d_draft_probs,
+                             void* d_workspace, size_t workspace_bytes, void* stream);
 
 /* ------------------------------------------------------------------------
  * One pipeline stage: the users of batch n (Sec. III-C, B_n(x)) verified
@@ -227,9 +236,10 @@ int dipsd_spec_verify_sparse(int B, const int* h_L, int V, int K, int logit_dtyp
  * may overlap an input buffer.
  *
  * Per-user tables cover all M users being served; h_members[b] (distinct, in
- * [0, M)) names the b-th user of this batch.  Per-batch tensors (d_q,
- * d_attn_out, logits, draft tokens, uniforms and the outputs) are packed in
- * h_members order exactly as for the two calls above.
+ * [0, M)) names the b-th user of this batch and is also its Philox key word
+ * 1 (its user id for dipsd_spec_verify).  Per-batch tensors (d_q,
+ * d_attn_out, logits, draft tokens and the outputs) are packed in h_members
+ * order exactly as for the two calls above.
  * h_L_all, h_ctx_all  [M] host;  d_block_table_all [M][max_blocks] int32.
  * ---------------------------------------------------------------------- */
 size_t dipsd_verify_batch_workspace_size(int B, const int* h_members, int M,
@@ -242,7 +252,7 @@ int dipsd_verify_batch(int B, const int* h_members, int M,
                        int Hq, int Hkv, int D, float softmax_scale, void* d_attn_out,
                        int V, int logit_dtype, const void* d_target_logits,
                        const void* d_draft_logits, const int* d_draft_tokens,
-                       const float* d_uniforms, int* d_accept_len, int* d_out_offsets,
+                       uint64_t seed, int* d_accept_len, int* d_out_offsets,
                        int* d_out_tokens, float* d_draft_probs,
                        void* d_workspace, size_t workspace_bytes, void* stream);
 
@@ -277,7 +287,7 @@ int dipsd_verify_batch_append(int B, const int* h_members, int M, const int* h_L
                               int Hq, int Hkv, int D, float softmax_scale, void* d_attn_out,
                               int V, int logit_dtype, const void* d_target_logits,
                               const void* d_draft_logits, const int* d_draft_tokens,
-                              const float* d_uniforms, int* d_accept_len, int* d_out_offsets,
+                              uint64_t seed, int* d_accept_len, int* d_out_offsets,
                               int* d_out_tokens, float* d_draft_probs, void* d_workspace,
                               size_t workspace_bytes, void* stream);
 
@@ -297,18 +307,66 @@ int dipsd_verify_batch_append(int B, const int* h_members, int M, const int* h_L
  * all (enough for bf16 logits with V up to about 160k at the maximum number of
  * positions); a larger batch is rejected with DIPSD_ERR_UNSUPPORTED before
  * anything is launched.  Every GPU that loads the library holds that 8 MiB
- * array until the process exits.  The first call on a device looks up the array's device address with
- * that device current; make that first call before any stream capture.  All
- * calls share the one array: calls that overlap on the GPU (other streams,
- * other host threads) race and must be serialised by the caller.  Each call
- * clears the array's status word on `stream` before its kernels run.
+ * array until the process exits.  The first call on a device looks up the
+ * array's device address with that device current; make that first call
+ * before any stream capture.  All calls share the one array: calls that
+ * overlap on the GPU (other streams, other host threads) race and must be
+ * serialised by the caller.  Each call clears the array's status word and
+ * arrival counters on `stream` before its kernels run, so no call depends
+ * on what an earlier one left there.  The device status bits
+ * (DIPSD_DEVERR_*) live in that array and cannot be read on this path: a
+ * draft token outside [0, V) is still treated as rejected, but unlike the
+ * workspace entry points nothing reports it.
  * ---------------------------------------------------------------------- */
 #define DIPSD_NOALLOC_MAX_POSITIONS 4096
-int dipsd_spec_verify_noalloc(int B, const int* h_L, int V, int logit_dtype,
-                              const void* d_target_logits, const void* d_draft_logits,
-                              const int* d_draft_tokens, const float* d_uniforms,
+int dipsd_spec_verify_noalloc(int B, const int* h_L, const int* h_user_id, uint64_t seed,
+                              int V, int logit_dtype, const void* d_target_logits,
+                              const void* d_draft_logits, const int* d_draft_tokens,
                               int* d_accept_len, int* d_out_offsets, int* d_out_tokens,
                               float* d_draft_probs, void* stream);
+
+/* ------------------------------------------------------------------------
+ * The random numbers of speculative sampling, written out (not in the paper:
+ * it leaves them unspecified; the generator is Philox4x64-10 of Salmon,
+ * Moraes, Dror and Shaw, SC 2011).
+ *
+ * dipsd_philox_words: words of counter blocks 0 .. n_blocks-1 of the stream
+ *   with key (seed, user_id): d_out[4 b + j] = word j of the block at
+ *   counter (b + 1, 0, 0, 0).  d_out: [4 n_blocks] uint64, 16-byte aligned;
+ *   user_id >= 0; 0 <= n_blocks <= 2^34.
+ * dipsd_verify_uniforms: the (u_acc, u_res) pairs dipsd_spec_verify draws
+ *   for this batch: d_uniforms [sum_i (L_i+1)][2] fp32, row q_off_i + t =
+ *   verify position t of user i (u_acc of a bonus position is drawn but
+ *   never used).  Arguments as for dipsd_spec_verify.
+ * Both are asynchronous on `stream` and allocate nothing.
+ * ---------------------------------------------------------------------- */
+int dipsd_philox_words(uint64_t seed, int user_id, long long n_blocks, uint64_t* d_out,
+                       void* stream);
+int dipsd_verify_uniforms(int B, const int* h_L, const int* h_user_id, uint64_t seed,
+                          float* d_uniforms, void* stream);
+
+/* ------------------------------------------------------------------------
+ * Test hooks (not for production use): process-wide overrides of the
+ * planners' choices, so that tests reach every kernel variant on small
+ * inputs.  Each override holds until it is set back to 0 (the planner's own
+ * choice).  The *_workspace_size calls plan with the same overrides, so set
+ * them before sizing a workspace.  The library never reads the environment.
+ *   DIPSD_TEST_ATTN_SPLIT_TILES  KV split length in 128-key tiles
+ *   DIPSD_TEST_ATTN_CLUSTER      cluster merge with this many splits (2..)
+ *   DIPSD_TEST_ATTN_PERSIST      1: persistent grid whenever allowed, 2: never
+ *   DIPSD_TEST_ATTN_GRID         persistent grid of at most this many CTAs
+ *   DIPSD_TEST_SPEC_NK1,
+ *   DIPSD_TEST_SPEC_NK2          16-byte vectors per lane in a segment of the
+ *                                two sampling passes (one of 16/8/4, 8/4/2)
+ * Returns DIPSD_ERR_INVALID_ARG for an unknown code or a negative value.
+ * ---------------------------------------------------------------------- */
+#define DIPSD_TEST_ATTN_SPLIT_TILES 1
+#define DIPSD_TEST_ATTN_CLUSTER 2
+#define DIPSD_TEST_ATTN_PERSIST 3
+#define DIPSD_TEST_ATTN_GRID 4
+#define DIPSD_TEST_SPEC_NK1 5
+#define DIPSD_TEST_SPEC_NK2 6
+int dipsd_test_set_override(int which, int value);
 
 #ifdef __cplusplus
 }

@@ -4,8 +4,8 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
-#include <cstdlib>
 #include <cstring>
 #include <mutex>
 #include <vector>
@@ -13,6 +13,7 @@
 #include "dipsd.h"
 #include "attention.cuh"
 #include "attention_tc.cuh"
+#include "philox.cuh"
 #include "spec_generic.cuh"
 #include "spec_verify.cuh"
 
@@ -29,6 +30,12 @@ constexpr int kCapSmall = 64;
 constexpr int kCapLarge = kMaxUsers;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Plan overrides set through dipsd_test_set_override (0 = the planner's own
+// choice); indexed by the DIPSD_TEST_* codes of dipsd.h.
+constexpr int kNumOverrides = 7;
+std::atomic<int> g_override[kNumOverrides];
+int plan_override(int which) { return g_override[which].load(std::memory_order_relaxed); }
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
 // ------------------------------------------------------------ device facts
@@ -182,9 +189,8 @@ void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int
   const int rows_cta = 128;
   const int slots = sms;
 
-  int forced = 0, forced_cluster = 0;
-  if (const char* e = std::getenv("DIPSD_ATTN_SPLIT_TILES")) forced = std::atoi(e);
-  if (const char* e = std::getenv("DIPSD_ATTN_CLUSTER")) forced_cluster = std::atoi(e);
+  const int forced = plan_override(DIPSD_TEST_ATTN_SPLIT_TILES);
+  const int forced_cluster = plan_override(DIPSD_TEST_ATTN_CLUSTER);
   const int cands[] = {1, 2, 3, 4, 5, 6, 8, 10, 12, 16, 20, 24, 32, 40, 48, 64, 96, 128, 192, 256, 384, 512, 1 << 30};
   // Costs in tile units: an item pays its tiles plus ~2 of prologue and
   // epilogue; splits merged by the separate merge kernel pay ~3 more (its
@@ -249,10 +255,8 @@ void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int
   // with the KV append (single-use patch barriers) nor the cluster merge.
   int persist_mode = -1;  // -1: by cost, 0: never, 1: whenever allowed
   int grid_cap = slots;
-  if (sms > 0) {  // forced for tests and tuning
-    if (const char* e = std::getenv("DIPSD_ATTN_PERSIST")) persist_mode = std::atoi(e) > 0 ? 1 : 0;
-    if (const char* e = std::getenv("DIPSD_ATTN_GRID")) grid_cap = std::max(1, std::min(slots, std::atoi(e)));
-  }
+  if (const int v = plan_override(DIPSD_TEST_ATTN_PERSIST)) persist_mode = v == 1 ? 1 : 0;
+  if (const int v = plan_override(DIPSD_TEST_ATTN_GRID)) grid_cap = std::max(1, std::min(slots, v));
   int best_pc = 0;
   double best_p = 1e300;
   if (persist_ok && pl.cluster <= 1 && persist_mode != 0) {
@@ -537,11 +541,10 @@ void plan_spec(int B, const int* L, int V, int elem, bool vec_ok, int sms, SpecP
     const int rows = pl.sum_t + (sparse ? 0 : pl.sum_l);
     int nk1 = pick_nk(kNk1, rows, pl.nvec, sms);
     int nk2 = sparse ? std::min(4, pick_nk(kNk2, B, pl.nvec, sms)) : pick_nk(kNk2, B, pl.nvec, sms);
-    if (sms > 0) {  // segment sizes forced for tests and tuning (never above the workspace bound)
-      if (const char* e = std::getenv("DIPSD_SPEC_NK1"))
-        for (int v : kNk1) if (v == std::atoi(e)) nk1 = v;
-      if (const char* e = std::getenv("DIPSD_SPEC_NK2"))
-        for (int v : kNk2) if (v == std::atoi(e) && !(sparse && v > 4)) nk2 = v;
+    if (sms > 0) {  // segment sizes set by a test override (never above the workspace bound)
+      const int o1 = plan_override(DIPSD_TEST_SPEC_NK1), o2 = plan_override(DIPSD_TEST_SPEC_NK2);
+      for (int v : kNk1) if (v == o1) nk1 = v;
+      for (int v : kNk2) if (v == o2 && !(sparse && v > 4)) nk2 = v;
     }
     const int nseg1 = ceil_div(pl.nvec, 32 * nk1), nseg2 = ceil_div(pl.nvec, 32 * nk2);
     const long long items1 = static_cast<long long>(rows) * nseg1;
@@ -642,12 +645,14 @@ struct SparseDraft {
 };
 
 template <int CAP>
-int run_spec_cap(const SpecPlan& pl, int dtype, const void* z, const void* w, const int* dt, const float* uni,
-                 int* acc, int* offs, int* toks, float* probs, unsigned* status, uint8_t* region,
+int run_spec_cap(const SpecPlan& pl, int dtype, const void* z, const void* w, const int* dt, uint64_t seed,
+                 const int* uid, int* acc, int* offs, int* toks, float* probs, unsigned* status, uint8_t* region,
                  cudaStream_t s, bool pdl, const SparseDraft& sd) {
   static thread_local SpecParams<CAP> p;
   std::memset(&p, 0, sizeof(p));
-  p.z = z; p.w = w; p.draft_tokens = dt; p.uniforms = uni;
+  p.z = z; p.w = w; p.draft_tokens = dt;
+  p.seed = seed;
+  for (int i = 0; i < pl.B; ++i) p.uid[i] = uid[i];
   p.stats = region;
   p.flags = region + pl.off_flags;
   p.part1 = reinterpret_cast<float4*>(region + pl.off_part1);
@@ -678,21 +683,31 @@ int run_spec_cap(const SpecPlan& pl, int dtype, const void* z, const void* w, co
   return pl.vec == 4 ? launch_spec_t<float, 4, CAP>(pl, p, s, pdl) : launch_spec_t<float, 1, CAP>(pl, p, s, pdl);
 }
 
-int run_spec(const SpecPlan& pl, int dtype, const void* z, const void* w, const int* dt, const float* uni,
-             int* acc, int* offs, int* toks, float* probs, unsigned* status, uint8_t* region, cudaStream_t s,
-             bool pdl, const SparseDraft& sd = SparseDraft{}) {
+int run_spec(const SpecPlan& pl, int dtype, const void* z, const void* w, const int* dt, uint64_t seed,
+             const int* uid, int* acc, int* offs, int* toks, float* probs, unsigned* status, uint8_t* region,
+             cudaStream_t s, bool pdl, const SparseDraft& sd = SparseDraft{}) {
   if (pl.B <= kCapSmall)
-    return run_spec_cap<kCapSmall>(pl, dtype, z, w, dt, uni, acc, offs, toks, probs, status, region, s, pdl, sd);
-  return run_spec_cap<kCapLarge>(pl, dtype, z, w, dt, uni, acc, offs, toks, probs, status, region, s, pdl, sd);
+    return run_spec_cap<kCapSmall>(pl, dtype, z, w, dt, seed, uid, acc, offs, toks, probs, status, region, s, pdl,
+                                   sd);
+  return run_spec_cap<kCapLarge>(pl, dtype, z, w, dt, seed, uid, acc, offs, toks, probs, status, region, s, pdl,
+                                 sd);
 }
 
-int check_spec_buffers(int dtype, const void* z, const void* w, const int* dt, const float* uni, int* acc,
-                       int* offs, int* toks, float* probs, int sum_l, int V, bool* vec_ok) {
+// Philox key word 1 of every user: a non-negative user id.
+int check_user_ids(int B, const int* uid) {
+  if (!uid) return DIPSD_ERR_INVALID_ARG;
+  for (int i = 0; i < B; ++i)
+    if (uid[i] < 0) return DIPSD_ERR_INVALID_ARG;
+  return DIPSD_OK;
+}
+
+int check_spec_buffers(int dtype, const void* z, const void* w, const int* dt, int* acc, int* offs, int* toks,
+                       float* probs, int sum_l, int V, bool* vec_ok) {
   if (dtype != DIPSD_BF16 && dtype != DIPSD_F32) return DIPSD_ERR_INVALID_ARG;
-  if (!z || !uni || !acc || !offs || !toks) return DIPSD_ERR_INVALID_ARG;
+  if (!z || !acc || !offs || !toks) return DIPSD_ERR_INVALID_ARG;
   if (sum_l > 0 && (!w || !dt)) return DIPSD_ERR_INVALID_ARG;
   const size_t elem = dtype == DIPSD_BF16 ? 2 : 4;
-  if (!aligned(z, elem) || (w && !aligned(w, elem)) || !aligned(uni, 8) || !aligned(acc, 4) ||
+  if (!aligned(z, elem) || (w && !aligned(w, elem)) || !aligned(acc, 4) ||
       !aligned(offs, 4) || !aligned(toks, 4) || (probs && !aligned(probs, 8)) || (dt && !aligned(dt, 4)))
     return DIPSD_ERR_INVALID_ARG;
   *vec_ok = (static_cast<size_t>(V) * elem) % 16 == 0 && aligned(z, 16) && (!w || aligned(w, 16));
@@ -752,6 +767,45 @@ const char* dipsd_status_string(int status) {
 int dipsd_abi_version(void) { return DIPSD_ABI_VERSION; }
 
 long long dipsd_launch_count(void) { return g_launches; }
+
+int dipsd_test_set_override(int which, int value) {
+  if (which < 1 || which >= kNumOverrides || value < 0) return DIPSD_ERR_INVALID_ARG;
+  g_override[which].store(value, std::memory_order_relaxed);
+  return DIPSD_OK;
+}
+
+int dipsd_philox_words(uint64_t seed, int user_id, long long n_blocks, uint64_t* d_out, void* stream) {
+  if (user_id < 0 || n_blocks < 0 || n_blocks > (1ll << 34) || (n_blocks > 0 && !d_out) || !aligned(d_out, 16))
+    return DIPSD_ERR_INVALID_ARG;
+  if (n_blocks == 0) return DIPSD_OK;
+  const long long grid = (n_blocks + 255) / 256;
+  if (launch(philox_words_kernel, dim3(static_cast<unsigned>(grid)), dim3(256), 0, static_cast<cudaStream_t>(stream),
+             0, false, static_cast<unsigned long long>(seed), static_cast<unsigned long long>(user_id), n_blocks,
+             reinterpret_cast<unsigned long long*>(d_out)) != cudaSuccess)
+    return DIPSD_ERR_CUDA;
+  return cuda_status();
+}
+
+int dipsd_verify_uniforms(int B, const int* h_L, const int* h_user_id, uint64_t seed, float* d_uniforms,
+                          void* stream) {
+  int st = check_spec_users(B, h_L, 1);
+  if (st != DIPSD_OK) return st;
+  st = check_user_ids(B, h_user_id);
+  if (st != DIPSD_OK) return st;
+  if (!d_uniforms || !aligned(d_uniforms, 8)) return DIPSD_ERR_INVALID_ARG;
+  static thread_local UniformParams p;
+  p.seed = seed;
+  p.B = B;
+  p.q_off[0] = 0;
+  for (int i = 0; i < B; ++i) {
+    p.q_off[i + 1] = p.q_off[i] + h_L[i] + 1;
+    p.uid[i] = h_user_id[i];
+  }
+  if (launch(verify_uniforms_kernel, dim3((p.q_off[B] + 255) / 256), dim3(256), 0, static_cast<cudaStream_t>(stream),
+             0, false, p, reinterpret_cast<float2*>(d_uniforms)) != cudaSuccess)
+    return DIPSD_ERR_CUDA;
+  return cuda_status();
+}
 
 // Attention workspace that covers the plans of both entry points (with and
 // without the KV append, which differ in their split choice).
@@ -837,16 +891,18 @@ size_t dipsd_spec_verify_workspace_size(int B, const int* h_L, int V) {
   return kHeaderBytes + spec_ws_need(B, h_L, V);
 }
 
-int dipsd_spec_verify(int B, const int* h_L, int V, int logit_dtype, const void* d_target_logits,
-                      const void* d_draft_logits, const int* d_draft_tokens, const float* d_uniforms,
+int dipsd_spec_verify(int B, const int* h_L, const int* h_user_id, uint64_t seed, int V, int logit_dtype,
+                      const void* d_target_logits, const void* d_draft_logits, const int* d_draft_tokens,
                       int* d_accept_len, int* d_out_offsets, int* d_out_tokens, float* d_draft_probs,
                       void* d_workspace, size_t workspace_bytes, void* stream) {
   int st = check_spec_users(B, h_L, V);
   if (st != DIPSD_OK) return st;
+  st = check_user_ids(B, h_user_id);
+  if (st != DIPSD_OK) return st;
   long long sum_l = 0;
   for (int i = 0; i < B; ++i) sum_l += h_L[i];
   bool vec_ok = false;
-  st = check_spec_buffers(logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
+  st = check_spec_buffers(logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_accept_len,
                           d_out_offsets, d_out_tokens, d_draft_probs, static_cast<int>(sum_l), V, &vec_ok);
   if (st != DIPSD_OK) return st;
   st = check_workspace(d_workspace, workspace_bytes, kHeaderBytes + spec_ws_need(B, h_L, V));
@@ -856,7 +912,7 @@ int dipsd_spec_verify(int B, const int* h_L, int V, int logit_dtype, const void*
   SpecPlan pl;
   plan_spec(B, h_L, V, logit_dtype == DIPSD_BF16 ? 2 : 4, vec_ok, f.sms, pl);
   uint8_t* ws = static_cast<uint8_t*>(d_workspace);
-  st = run_spec(pl, logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
+  st = run_spec(pl, logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, seed, h_user_id, d_accept_len,
                 d_out_offsets, d_out_tokens, d_draft_probs, reinterpret_cast<unsigned*>(ws), ws + kHeaderBytes,
                 static_cast<cudaStream_t>(stream), true);
   return st != DIPSD_OK ? st : cuda_status();
@@ -868,19 +924,21 @@ size_t dipsd_spec_verify_sparse_workspace_size(int B, const int* h_L, int V) {
   return need ? kHeaderBytes + need : 0;
 }
 
-int dipsd_spec_verify_sparse(int B, const int* h_L, int V, int K, int logit_dtype, const void* d_target_logits,
-                             const int* d_draft_tokens, const float* d_draft_logq, const int* d_topk_idx,
-                             const float* d_topk_q, const float* d_uniforms, int* d_accept_len, int* d_out_offsets,
-                             int* d_out_tokens, float* d_draft_probs, void* d_workspace, size_t workspace_bytes,
-                             void* stream) {
+int dipsd_spec_verify_sparse(int B, const int* h_L, const int* h_user_id, uint64_t seed, int V, int K,
+                             int logit_dtype, const void* d_target_logits, const int* d_draft_tokens,
+                             const float* d_draft_logq, const int* d_topk_idx, const float* d_topk_q,
+                             int* d_accept_len, int* d_out_offsets, int* d_out_tokens, float* d_draft_probs,
+                             void* d_workspace, size_t workspace_bytes, void* stream) {
   int st = check_spec_users(B, h_L, V);
+  if (st != DIPSD_OK) return st;
+  st = check_user_ids(B, h_user_id);
   if (st != DIPSD_OK) return st;
   if (K < 1 || K > kMaxTopK) return DIPSD_ERR_INVALID_ARG;
   long long sum_l = 0;
   for (int i = 0; i < B; ++i) sum_l += h_L[i];
   bool vec_ok = false;
   // (the draft-logits slot is checked with the target logits' pointer: the sparse path has none)
-  st = check_spec_buffers(logit_dtype, d_target_logits, d_target_logits, d_draft_tokens, d_uniforms, d_accept_len,
+  st = check_spec_buffers(logit_dtype, d_target_logits, d_target_logits, d_draft_tokens, d_accept_len,
                           d_out_offsets, d_out_tokens, d_draft_probs, static_cast<int>(sum_l), V, &vec_ok);
   if (st != DIPSD_OK) return st;
   if (sum_l > 0 && (!d_draft_logq || !d_topk_idx || !d_topk_q || !aligned(d_draft_logq, 4) ||
@@ -899,17 +957,19 @@ int dipsd_spec_verify_sparse(int B, const int* h_L, int V, int K, int logit_dtyp
   sd.topk_q = d_topk_q;
   sd.topk = K;
   uint8_t* ws = static_cast<uint8_t*>(d_workspace);
-  st = run_spec(pl, logit_dtype, d_target_logits, nullptr, d_draft_tokens, d_uniforms, d_accept_len, d_out_offsets,
-                d_out_tokens, d_draft_probs, reinterpret_cast<unsigned*>(ws), ws + kHeaderBytes,
+  st = run_spec(pl, logit_dtype, d_target_logits, nullptr, d_draft_tokens, seed, h_user_id, d_accept_len,
+                d_out_offsets, d_out_tokens, d_draft_probs, reinterpret_cast<unsigned*>(ws), ws + kHeaderBytes,
                 static_cast<cudaStream_t>(stream), true, sd);
   return st != DIPSD_OK ? st : cuda_status();
 }
 
-int dipsd_spec_verify_noalloc(int B, const int* h_L, int V, int logit_dtype, const void* d_target_logits,
-                              const void* d_draft_logits, const int* d_draft_tokens, const float* d_uniforms,
+int dipsd_spec_verify_noalloc(int B, const int* h_L, const int* h_user_id, uint64_t seed, int V, int logit_dtype,
+                              const void* d_target_logits, const void* d_draft_logits, const int* d_draft_tokens,
                               int* d_accept_len, int* d_out_offsets, int* d_out_tokens, float* d_draft_probs,
                               void* stream) {
   int st = check_spec_users(B, h_L, V);
+  if (st != DIPSD_OK) return st;
+  st = check_user_ids(B, h_user_id);
   if (st != DIPSD_OK) return st;
   long long sum_l = 0, sum_t = 0;
   for (int i = 0; i < B; ++i) {
@@ -918,7 +978,7 @@ int dipsd_spec_verify_noalloc(int B, const int* h_L, int V, int logit_dtype, con
   }
   if (sum_t > DIPSD_NOALLOC_MAX_POSITIONS) return DIPSD_ERR_UNSUPPORTED;
   bool vec_ok = false;
-  st = check_spec_buffers(logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
+  st = check_spec_buffers(logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_accept_len,
                           d_out_offsets, d_out_tokens, d_draft_probs, static_cast<int>(sum_l), V, &vec_ok);
   if (st != DIPSD_OK) return st;
   DeviceFacts f;
@@ -929,8 +989,10 @@ int dipsd_spec_verify_noalloc(int B, const int* h_L, int V, int logit_dtype, con
   uint8_t* ws = noalloc_scratch();
   if (!ws) return DIPSD_ERR_CUDA;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (cudaMemsetAsync(ws, 0, kStatusBytes, s) != cudaSuccess) return DIPSD_ERR_CUDA;
-  st = run_spec(pl, logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
+  // the status word and every arrival counter start at zero, whatever an
+  // earlier call left there
+  if (cudaMemsetAsync(ws, 0, kHeaderBytes, s) != cudaSuccess) return DIPSD_ERR_CUDA;
+  st = run_spec(pl, logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, seed, h_user_id, d_accept_len,
                 d_out_offsets, d_out_tokens, d_draft_probs, reinterpret_cast<unsigned*>(ws), ws + kHeaderBytes, s,
                 true);
   return st != DIPSD_OK ? st : cuda_status();
@@ -969,7 +1031,7 @@ static int verify_batch_impl(int B, const int* h_members, int M, const int* h_L_
                              const int* d_block_table_all, int max_blocks, int Hq, int Hkv, int D,
                              float softmax_scale, void* d_attn_out, int V, int logit_dtype,
                              const void* d_target_logits, const void* d_draft_logits, const int* d_draft_tokens,
-                             const float* d_uniforms, int* d_accept_len, int* d_out_offsets, int* d_out_tokens,
+                             uint64_t seed, int* d_accept_len, int* d_out_offsets, int* d_out_tokens,
                              float* d_draft_probs, void* d_workspace, size_t workspace_bytes, void* stream,
                              const KvAppend& app) {
   std::vector<int> L, ctx;
@@ -985,7 +1047,7 @@ static int verify_batch_impl(int B, const int* h_members, int M, const int* h_L_
   long long sum_l = 0;
   for (int b = 0; b < B; ++b) sum_l += L[b];
   bool vec_ok = false;
-  st = check_spec_buffers(logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
+  st = check_spec_buffers(logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_accept_len,
                           d_out_offsets, d_out_tokens, d_draft_probs, static_cast<int>(sum_l), V, &vec_ok);
   if (st != DIPSD_OK) return st;
   DeviceFacts f;
@@ -1005,7 +1067,8 @@ static int verify_batch_impl(int B, const int* h_members, int M, const int* h_L_
   // (so everything before this call is complete), streams the KV cache
   // while the sampling kernel's per-user descents finish, and waits for
   // that kernel only before it exits.
-  st = run_spec(sp, logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len,
+  // each member's Philox key word 1 is its index in the per-user tables
+  st = run_spec(sp, logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, seed, h_members, d_accept_len,
                 d_out_offsets, d_out_tokens, d_draft_probs, status, ws + kHeaderBytes + attn_region, s, true);
   if (st != DIPSD_OK) return st;
   st = run_attention(ap, d_q, d_k_cache, d_v_cache, num_blocks, d_block_table_all, max_blocks, softmax_scale,
@@ -1017,12 +1080,12 @@ int dipsd_verify_batch(int B, const int* h_members, int M, const int* h_L_all, c
                        const void* d_q, const void* d_k_cache, const void* d_v_cache, int num_blocks,
                        const int* d_block_table_all, int max_blocks, int Hq, int Hkv, int D, float softmax_scale,
                        void* d_attn_out, int V, int logit_dtype, const void* d_target_logits,
-                       const void* d_draft_logits, const int* d_draft_tokens, const float* d_uniforms,
+                       const void* d_draft_logits, const int* d_draft_tokens, uint64_t seed,
                        int* d_accept_len, int* d_out_offsets, int* d_out_tokens, float* d_draft_probs,
                        void* d_workspace, size_t workspace_bytes, void* stream) {
   return verify_batch_impl(B, h_members, M, h_L_all, h_ctx_all, d_q, d_k_cache, d_v_cache, num_blocks,
                            d_block_table_all, max_blocks, Hq, Hkv, D, softmax_scale, d_attn_out, V, logit_dtype,
-                           d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len, d_out_offsets,
+                           d_target_logits, d_draft_logits, d_draft_tokens, seed, d_accept_len, d_out_offsets,
                            d_out_tokens, d_draft_probs, d_workspace, workspace_bytes, stream, KvAppend{});
 }
 
@@ -1031,7 +1094,7 @@ int dipsd_verify_batch_append(int B, const int* h_members, int M, const int* h_L
                               void* d_v_cache, int num_blocks, const int* d_block_table_all, int max_blocks, int Hq,
                               int Hkv, int D, float softmax_scale, void* d_attn_out, int V, int logit_dtype,
                               const void* d_target_logits, const void* d_draft_logits, const int* d_draft_tokens,
-                              const float* d_uniforms, int* d_accept_len, int* d_out_offsets, int* d_out_tokens,
+                              uint64_t seed, int* d_accept_len, int* d_out_offsets, int* d_out_tokens,
                               float* d_draft_probs, void* d_workspace, size_t workspace_bytes, void* stream) {
   const int st = check_append(d_new_k, d_new_v, d_q);
   if (st != DIPSD_OK) return st;
@@ -1040,7 +1103,7 @@ int dipsd_verify_batch_append(int B, const int* h_members, int M, const int* h_L
   app.new_v = d_new_v;
   return verify_batch_impl(B, h_members, M, h_L_all, h_ctx_all, d_q, d_k_cache, d_v_cache, num_blocks,
                            d_block_table_all, max_blocks, Hq, Hkv, D, softmax_scale, d_attn_out, V, logit_dtype,
-                           d_target_logits, d_draft_logits, d_draft_tokens, d_uniforms, d_accept_len, d_out_offsets,
+                           d_target_logits, d_draft_logits, d_draft_tokens, seed, d_accept_len, d_out_offsets,
                            d_out_tokens, d_draft_probs, d_workspace, workspace_bytes, stream, app);
 }
 

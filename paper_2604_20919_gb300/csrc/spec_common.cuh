@@ -4,6 +4,7 @@
 #pragma once
 
 #include "common.cuh"
+#include "philox.cuh"
 
 namespace dipsd {
 
@@ -25,7 +26,6 @@ struct SpecParams {
   const void* z;              // target logits [sum T][V]
   const void* w;              // draft logits  [sum L][V]
   const int* draft_tokens;    // [sum L]
-  const float* uniforms;      // [sum T][2]
   void* stats;                // [sum T] row statistics (layout private to each path)
   unsigned char* flags;       // [sum T]: acceptance bit
   float* draft_probs;         // optional [sum T][2]
@@ -45,8 +45,10 @@ struct SpecParams {
   unsigned* counters;  // [kCounterWords], zero between calls
   int sum_t, nseg1, nseg2, n_items1, n_items2;
   int B, V, nvec;             // nvec = V / VEC
+  unsigned long long seed;    // Philox key word 0 (the caller's seed)
   int q_off[CAP + 1];         // first verify position of user i
   int l_off[CAP + 1];         // first draft row of user i
+  int uid[CAP];               // Philox key word 1 of user i (its user id)
 };
 
 // ----------------------------------------------------- row element access

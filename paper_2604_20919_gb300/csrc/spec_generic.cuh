@@ -1,5 +1,7 @@
-// spec_verify, generic path: used when a logit row is not 16-byte aligned or a
-// row slice would not fit the shared-memory staging of spec_verify.cuh.
+// spec_verify, generic path: used when a logit row is not 16-byte aligned
+// (V times the element size not a multiple of 16 bytes, or a row pointer off
+// a 16-byte boundary), where the register path's 16-byte vector loads do not
+// apply, or when a row has more segments than its arrival counters can count.
 // Same arithmetic contract (speculative sampling, Sec. II-A stage 2); rows are
 // streamed with per-thread loads instead of staged.
 //
@@ -136,7 +138,7 @@ spec_stats_generic_kernel(const __grid_constant__ SpecParams<CAP> p) {
     if (d >= 0 && d < p.V) {
       pd = expf(load_elem<T>(zrow, d) - a.x) / a.y;
       qd = expf(load_elem<T>(wrow_p, d) - a.z) / a.w;
-      flag = p.uniforms[2 * n] * qd < pd ? 1 : 0;
+      flag = verify_uniforms(p.seed, static_cast<unsigned>(p.uid[ui]), t).x * qd < pd ? 1 : 0;
     } else {
       atomicOr(p.status, kDevErrBadToken);
     }
@@ -194,7 +196,7 @@ spec_sample_generic_kernel(const __grid_constant__ SpecParams<CAP> p) {
   const float4 st = static_cast<const float4*>(p.stats)[n];
   const T* zrow = static_cast<const T*>(p.z) + static_cast<size_t>(n) * p.V;
   const T* wrow = static_cast<const T*>(p.w) + static_cast<size_t>(a < Li ? l0 + a : 0) * p.V;
-  const float u = p.uniforms[2 * n + 1];
+  const float u = verify_uniforms(p.seed, static_cast<unsigned>(p.uid[ui]), a).y;
   const float inv_z = 1.f / st.y, inv_w = 1.f / st.w;
   bool residual = a < Li;
 

@@ -501,7 +501,7 @@ __device__ __forceinline__ void vec_weights_table(const uint4& rz, const float (
 // position writes a_i.  One thread.
 template <int CAP, bool SP>
 __device__ __forceinline__ void decide_from_sums(const SpecParams<CAP>& p, int ui, int t, RefSum az, RefSum aw,
-                                                 float zd, float wd, float logq) {
+                                                 float zd, float wd, float logq, float u) {
   const int q0 = p.q_off[ui];
   const int Li = p.q_off[ui + 1] - q0 - 1;
   const int n = q0 + t;
@@ -518,7 +518,6 @@ __device__ __forceinline__ void decide_from_sums(const SpecParams<CAP>& p, int u
     st.khi = st.klo = 0.f;
     float pd = 0.f, qd = 0.f;
     unsigned char flag = 0;
-    const float u = p.uniforms[2 * n];
     if (has_q && SP) {
       // sparse payload: q(d) is given; the residual scales q by sz, kept as
       // a float-float pair
@@ -590,6 +589,8 @@ __device__ __forceinline__ void decide_position(const SpecParams<CAP>& p, int ui
     else wd = __ldcg(&pw->w);
   }
   RefSum az{kEmptyRef, FF{0.f, 0.f}}, aw{kEmptyRef, FF{0.f, 0.f}};
+  // the acceptance uniform (independent of the loads, so it overlaps them)
+  const float u_acc = has_q ? verify_uniforms(p.seed, static_cast<unsigned>(p.uid[ui]), t).x : 0.f;
 #pragma unroll 2
   for (int sg = lane; sg < p.nseg1; sg += 32) {
     const float4 vz = __ldcg(pz + sg);
@@ -601,7 +602,7 @@ __device__ __forceinline__ void decide_position(const SpecParams<CAP>& p, int ui
   if (has_q && !SP) aw = warp_refsum(aw);
   if (lane == 0) {
     p.counters[n] = 0u;
-    decide_from_sums<CAP, SP>(p, ui, t, az, aw, zd, wd, logq);
+    decide_from_sums<CAP, SP>(p, ui, t, az, aw, zd, wd, logq, u_acc);
   }
 }
 
@@ -667,8 +668,7 @@ __device__ __forceinline__ void descend(const SpecParams<CAP>& p, int ui, int a,
                                         const T* zrow, const T* wrow, const int (&sidx)[2], const float (&sq)[2],
                                         int lane) {
   constexpr int N = Vec16<T>::N;
-  const int q0 = p.q_off[ui], l0 = p.l_off[ui];
-  const int n = q0 + a;
+  const int l0 = p.l_off[ui];
   const float4* part = p.part2 + static_cast<size_t>(ui) * p.nseg2;
   const int per = (p.nseg2 + 31) >> 5;  // lane j owns segments [j per, (j + 1) per)
   const int s0 = lane * per;
@@ -690,7 +690,7 @@ __device__ __forceinline__ void descend(const SpecParams<CAP>& p, int ui, int a,
   const int mode0 = residual ? 0 : 1;
   float2 v[kRun];
   load_run(mode0, v);
-  const float u = p.uniforms[2 * n + 1];
+  const float u = verify_uniforms(p.seed, static_cast<unsigned>(p.uid[ui]), a).y;
   const int dtok = lane < a ? p.draft_tokens[l0 + lane] : 0;  // a <= L_i <= 31
   int o = 0;
   for (int j = lane; j < ui; j += 32)

@@ -8,6 +8,7 @@ back to anything else.
 """
 from __future__ import annotations
 
+import contextlib
 import ctypes
 import os
 from typing import Optional, Sequence
@@ -35,14 +36,19 @@ EXPORTS = (
     "dipsd_verify_batch_workspace_size", "dipsd_verify_batch", "dipsd_spec_verify_noalloc",
     "dipsd_verify_attention_append", "dipsd_verify_batch_append",
     "dipsd_spec_verify_sparse_workspace_size", "dipsd_spec_verify_sparse", "dipsd_verify_attention_plan",
+    "dipsd_philox_words", "dipsd_verify_uniforms", "dipsd_test_set_override",
 )
 NOALLOC_MAX_POSITIONS = 4096
+# dipsd_test_set_override codes
+TEST_OVERRIDES = {"attn_split_tiles": 1, "attn_cluster": 2, "attn_persist": 3, "attn_grid": 4,
+                  "spec_nk1": 5, "spec_nk2": 6}
 
 _lib: Optional[ctypes.CDLL] = None
 _i32p = ctypes.POINTER(ctypes.c_int)
 _vp = ctypes.c_void_p
 _sz = ctypes.c_size_t
 _i = ctypes.c_int
+_u64 = ctypes.c_uint64
 
 
 class AttentionPlan(ctypes.Structure):
@@ -76,30 +82,38 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.dipsd_spec_verify_workspace_size.restype = _sz
     lib.dipsd_spec_verify_workspace_size.argtypes = [_i, _i32p, _i]
     lib.dipsd_spec_verify.restype = _i
-    lib.dipsd_spec_verify.argtypes = [_i, _i32p, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
+    lib.dipsd_spec_verify.argtypes = [_i, _i32p, _i32p, _u64, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz,
+                                      _vp]
     lib.dipsd_verify_batch_workspace_size.restype = _sz
     lib.dipsd_verify_batch_workspace_size.argtypes = [_i, _i32p, _i, _i32p, _i32p, _i, _i, _i, _i]
     lib.dipsd_verify_batch.restype = _i
     lib.dipsd_verify_batch.argtypes = [_i, _i32p, _i, _i32p, _i32p, _vp, _vp, _vp, _i, _vp, _i, _i, _i, _i,
-                                       ctypes.c_float, _vp, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                       ctypes.c_float, _vp, _i, _i, _vp, _vp, _vp, _u64, _vp, _vp, _vp, _vp,
                                        _vp, _sz, _vp]
     lib.dipsd_verify_attention_append.restype = _i
     lib.dipsd_verify_attention_append.argtypes = [_i, _i32p, _i32p, _vp, _vp, _vp, _vp, _vp, _i, _vp, _i, _i, _i,
                                                   _i, ctypes.c_float, _vp, _vp, _sz, _vp]
     lib.dipsd_verify_batch_append.restype = _i
     lib.dipsd_verify_batch_append.argtypes = [_i, _i32p, _i, _i32p, _i32p, _vp, _vp, _vp, _vp, _vp, _i, _vp, _i,
-                                              _i, _i, _i, ctypes.c_float, _vp, _i, _i, _vp, _vp, _vp, _vp, _vp,
+                                              _i, _i, _i, ctypes.c_float, _vp, _i, _i, _vp, _vp, _vp, _u64, _vp,
                                               _vp, _vp, _vp, _vp, _sz, _vp]
     lib.dipsd_spec_verify_sparse_workspace_size.restype = _sz
     lib.dipsd_spec_verify_sparse_workspace_size.argtypes = [_i, _i32p, _i]
     lib.dipsd_spec_verify_sparse.restype = _i
-    lib.dipsd_spec_verify_sparse.argtypes = [_i, _i32p, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
-                                             _vp, _sz, _vp]
+    lib.dipsd_spec_verify_sparse.argtypes = [_i, _i32p, _i32p, _u64, _i, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                             _vp, _vp, _vp, _sz, _vp]
     lib.dipsd_verify_attention_plan.restype = _i
     lib.dipsd_verify_attention_plan.argtypes = [_i, _i32p, _i32p, _i, _i, _i, _i, _i,
                                                 ctypes.POINTER(AttentionPlan), _i32p, _i32p]
     lib.dipsd_spec_verify_noalloc.restype = _i
-    lib.dipsd_spec_verify_noalloc.argtypes = [_i, _i32p, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]
+    lib.dipsd_spec_verify_noalloc.argtypes = [_i, _i32p, _i32p, _u64, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                              _vp]
+    lib.dipsd_philox_words.restype = _i
+    lib.dipsd_philox_words.argtypes = [_u64, _i, ctypes.c_longlong, _vp, _vp]
+    lib.dipsd_verify_uniforms.restype = _i
+    lib.dipsd_verify_uniforms.argtypes = [_i, _i32p, _i32p, _u64, _vp, _vp]
+    lib.dipsd_test_set_override.restype = _i
+    lib.dipsd_test_set_override.argtypes = [_i, _i]
     _lib = lib
     return lib
 
@@ -107,6 +121,20 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
 def dipsd_launch_count() -> int:
     """Kernels launched by the library from this host thread so far."""
     return int(load().dipsd_launch_count())
+
+
+@contextlib.contextmanager
+def plan_override(**overrides):
+    """Test hook: plan overrides (names of TEST_OVERRIDES, 0 = the planner's
+    own choice) held for the duration of the block, process-wide."""
+    lib = load()
+    for k, v in overrides.items():
+        _check(lib.dipsd_test_set_override(TEST_OVERRIDES[k], int(v)), "dipsd_test_set_override")
+    try:
+        yield
+    finally:
+        for k in overrides:
+            lib.dipsd_test_set_override(TEST_OVERRIDES[k], 0)
 
 
 def status_string(status: int) -> str:
@@ -255,25 +283,54 @@ def spec_outputs(L, device, with_probs=True):
             torch.empty(sum_t, 2, dtype=torch.float32, device=device) if with_probs else None)
 
 
-def dipsd_spec_verify(L, target_logits, draft_logits, draft_tokens, uniforms, outputs=None, ws=None,
+def _user_ids(user_ids, B):
+    u, pu = _host_i32(user_ids)
+    if u.shape != (B,):
+        raise ValueError("user_ids must hold one id per user")
+    return u, pu
+
+
+def dipsd_philox_words(seed: int, user_id: int, n_blocks: int, out=None, stream=None) -> torch.Tensor:
+    """Words of counter blocks 0 .. n_blocks-1 of the Philox4x64-10 stream with
+    key (seed, user_id), as int64 bit patterns [n_blocks * 4] on the current device."""
+    if out is None:
+        out = torch.empty(4 * int(n_blocks), dtype=torch.int64, device="cuda")
+    _check(load().dipsd_philox_words(int(seed), int(user_id), int(n_blocks), _dptr(out, "out", torch.int64),
+                                     _stream(stream)), "dipsd_philox_words")
+    return out
+
+
+def dipsd_verify_uniforms(L, user_ids, seed: int, out=None, stream=None) -> torch.Tensor:
+    """The (u_acc, u_res) pairs spec verification draws for this batch, [sum T][2] fp32."""
+    a, pa = _host_i32(L)
+    u, pu = _user_ids(user_ids, len(a))
+    if out is None:
+        out = torch.empty(int((a + 1).sum()), 2, dtype=torch.float32, device="cuda")
+    _check(load().dipsd_verify_uniforms(len(a), pa, pu, int(seed), _dptr(out, "out", torch.float32),
+                                        _stream(stream)), "dipsd_verify_uniforms")
+    return out
+
+
+def dipsd_spec_verify(L, user_ids, seed, target_logits, draft_logits, draft_tokens, outputs=None, ws=None,
                       stream=None):
-    """Speculative verification; returns (accept_len, out_offsets, out_tokens, draft_probs)."""
+    """Speculative verification with in-kernel Philox uniforms keyed on
+    (seed, user_ids[i]); returns (accept_len, out_offsets, out_tokens, draft_probs)."""
     lib = load()
     a, pa = _host_i32(L)
+    u, pu = _user_ids(user_ids, len(a))
     sum_t, sum_l = int((a + 1).sum()), int(a.sum())
     V = target_logits.shape[1]
     dt = _logit_dtype(target_logits)
-    if target_logits.shape[0] != sum_t or tuple(uniforms.shape) != (sum_t, 2):
-        raise ValueError("target_logits / uniforms do not match the draft lengths")
+    if target_logits.shape[0] != sum_t:
+        raise ValueError("target_logits do not match the draft lengths")
     if draft_logits.shape != (sum_l, V) or draft_logits.dtype != target_logits.dtype or draft_tokens.numel() != sum_l:
         raise ValueError("draft_logits / draft_tokens do not match the draft lengths")
     acc, offs, toks, probs = outputs if outputs is not None else spec_outputs(a, target_logits.device)
     if ws is None:
         ws = workspace(dipsd_spec_verify_workspace_size(a, V), target_logits.device)
-    st = lib.dipsd_spec_verify(len(a), pa, V, dt, _dptr(target_logits, "target_logits"),
+    st = lib.dipsd_spec_verify(len(a), pa, pu, int(seed), V, dt, _dptr(target_logits, "target_logits"),
                                _dptr(draft_logits, "draft_logits") if sum_l else 0,
                                _dptr(draft_tokens, "draft_tokens", torch.int32) if sum_l else 0,
-                               _dptr(uniforms, "uniforms", torch.float32),
                                _dptr(acc, "accept_len", torch.int32), _dptr(offs, "out_offsets", torch.int32),
                                _dptr(toks, "out_tokens", torch.int32),
                                _dptr(probs, "draft_probs", torch.float32), _dptr(ws, "workspace"), ws.numel(),
@@ -287,30 +344,30 @@ def dipsd_spec_verify_sparse_workspace_size(L, V: int) -> int:
     return int(load().dipsd_spec_verify_sparse_workspace_size(len(a), pa, V))
 
 
-def dipsd_spec_verify_sparse(L, target_logits, draft_tokens, draft_logq, topk_idx, topk_q, uniforms, outputs=None,
-                             ws=None, stream=None):
+def dipsd_spec_verify_sparse(L, user_ids, seed, target_logits, draft_tokens, draft_logq, topk_idx, topk_q,
+                             outputs=None, ws=None, stream=None):
     """Speculative verification from a sparse draft payload; returns
     (accept_len, out_offsets, out_tokens, draft_probs)."""
     lib = load()
     a, pa = _host_i32(L)
+    u, pu = _user_ids(user_ids, len(a))
     sum_t, sum_l = int((a + 1).sum()), int(a.sum())
     V = target_logits.shape[1]
     K = int(topk_idx.shape[1]) if topk_idx.dim() == 2 else 0
-    if target_logits.shape[0] != sum_t or tuple(uniforms.shape) != (sum_t, 2):
-        raise ValueError("target_logits / uniforms do not match the draft lengths")
+    if target_logits.shape[0] != sum_t:
+        raise ValueError("target_logits do not match the draft lengths")
     if (draft_tokens.numel() != sum_l or draft_logq.numel() != sum_l or tuple(topk_idx.shape) != (sum_l, K)
             or tuple(topk_q.shape) != (sum_l, K)):
         raise ValueError("draft tokens / log-probabilities / table do not match the draft lengths")
     acc, offs, toks, probs = outputs if outputs is not None else spec_outputs(a, target_logits.device)
     if ws is None:
         ws = workspace(dipsd_spec_verify_sparse_workspace_size(a, V), target_logits.device)
-    st = lib.dipsd_spec_verify_sparse(len(a), pa, V, max(K, 1), _logit_dtype(target_logits),
+    st = lib.dipsd_spec_verify_sparse(len(a), pa, pu, int(seed), V, max(K, 1), _logit_dtype(target_logits),
                                       _dptr(target_logits, "target_logits"),
                                       _dptr(draft_tokens, "draft_tokens", torch.int32) if sum_l else 0,
                                       _dptr(draft_logq, "draft_logq", torch.float32) if sum_l else 0,
                                       _dptr(topk_idx, "topk_idx", torch.int32) if sum_l else 0,
                                       _dptr(topk_q, "topk_q", torch.float32) if sum_l else 0,
-                                      _dptr(uniforms, "uniforms", torch.float32),
                                       _dptr(acc, "accept_len", torch.int32), _dptr(offs, "out_offsets", torch.int32),
                                       _dptr(toks, "out_tokens", torch.int32),
                                       _dptr(probs, "draft_probs", torch.float32), _dptr(ws, "workspace"), ws.numel(),
@@ -328,7 +385,7 @@ def dipsd_verify_batch_workspace_size(members, L_all, ctx_all, Hq, Hkv, D, V) ->
 
 
 def _verify_batch(members, L_all, ctx_all, q, k_cache, v_cache, block_table_all, softmax_scale, target_logits,
-                  draft_logits, draft_tokens, uniforms, attn_out, outputs, ws, stream, new_kv):
+                  draft_logits, draft_tokens, seed, attn_out, outputs, ws, stream, new_kv):
     """Attention then speculative verification for the users `members` of one stage.
 
     Returns (attn_out, accept_len, out_offsets, out_tokens, draft_probs).
@@ -343,8 +400,8 @@ def _verify_batch(members, L_all, ctx_all, q, k_cache, v_cache, block_table_all,
     Hq, V = q.shape[1], target_logits.shape[1]
     if page != PAGE_SIZE or tuple(q.shape) != (sum_t, Hq, D):
         raise ValueError("q does not match the members' draft lengths")
-    if target_logits.shape[0] != sum_t or draft_logits.shape != (sum_l, V) or tuple(uniforms.shape) != (sum_t, 2):
-        raise ValueError("logits / uniforms do not match the members' draft lengths")
+    if target_logits.shape[0] != sum_t or draft_logits.shape != (sum_l, V):
+        raise ValueError("logits do not match the members' draft lengths")
     if attn_out is None:
         attn_out = torch.empty_like(q)
     acc, offs, toks, probs = outputs if outputs is not None else spec_outputs(Lb, q.device)
@@ -366,8 +423,7 @@ def _verify_batch(members, L_all, ctx_all, q, k_cache, v_cache, block_table_all,
                                 Hq, Hkv, D, float(softmax_scale), _dptr(attn_out, "attn_out", torch.bfloat16), V,
                                 _logit_dtype(target_logits), _dptr(target_logits, "target_logits"),
                                 _dptr(draft_logits, "draft_logits") if sum_l else 0,
-                                _dptr(draft_tokens, "draft_tokens", torch.int32) if sum_l else 0,
-                                _dptr(uniforms, "uniforms", torch.float32),
+                                _dptr(draft_tokens, "draft_tokens", torch.int32) if sum_l else 0, int(seed),
                                 _dptr(acc, "accept_len", torch.int32), _dptr(offs, "out_offsets", torch.int32),
                                 _dptr(toks, "out_tokens", torch.int32), _dptr(probs, "draft_probs", torch.float32),
                                 _dptr(ws, "workspace"), ws.numel(), _stream(stream))
@@ -376,20 +432,21 @@ def _verify_batch(members, L_all, ctx_all, q, k_cache, v_cache, block_table_all,
 
 
 def dipsd_verify_batch(members, L_all, ctx_all, q, k_cache, v_cache, block_table_all, softmax_scale,
-                       target_logits, draft_logits, draft_tokens, uniforms, attn_out=None, outputs=None,
+                       target_logits, draft_logits, draft_tokens, seed, attn_out=None, outputs=None,
                        ws=None, stream=None):
-    """Attention then speculative verification for the users `members` of one stage.
+    """Attention then speculative verification for the users `members` of one
+    stage (each member's Philox key is (seed, member index)).
 
     Returns (attn_out, accept_len, out_offsets, out_tokens, draft_probs).
     """
     return _verify_batch(members, L_all, ctx_all, q, k_cache, v_cache, block_table_all, softmax_scale,
-                         target_logits, draft_logits, draft_tokens, uniforms, attn_out, outputs, ws, stream, None)
+                         target_logits, draft_logits, draft_tokens, seed, attn_out, outputs, ws, stream, None)
 
 
 def dipsd_verify_batch_append(members, L_all, ctx_all, q, new_k, new_v, k_cache, v_cache, block_table_all,
-                              softmax_scale, target_logits, draft_logits, draft_tokens, uniforms, attn_out=None,
+                              softmax_scale, target_logits, draft_logits, draft_tokens, seed, attn_out=None,
                               outputs=None, ws=None, stream=None):
     """As dipsd_verify_batch, first writing the verify tokens' K/V rows into their pages."""
     return _verify_batch(members, L_all, ctx_all, q, k_cache, v_cache, block_table_all, softmax_scale,
-                         target_logits, draft_logits, draft_tokens, uniforms, attn_out, outputs, ws, stream,
+                         target_logits, draft_logits, draft_tokens, seed, attn_out, outputs, ws, stream,
                          (new_k, new_v))

@@ -32,7 +32,7 @@ def test_header_declarations_are_exported(lib):
 
 
 def test_status_strings_and_version(lib):
-    assert lib.dipsd_abi_version() == 1
+    assert lib.dipsd_abi_version() == 2
     from paper_2604_20919_gb300 import dipsd
     assert dipsd.status_string(0) == "ok"
     assert "invalid" in dipsd.status_string(1)
@@ -76,21 +76,68 @@ def test_attention_rejects_null_and_misaligned_pointers(lib):
 
 
 def test_spec_verify_rejects_bad_arguments(lib):
+    u, pu = _i32([0, 1])
     a, pa = _i32([2, 40])
-    assert lib.dipsd_spec_verify(2, pa, 100, 0, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, 1 << 20,
+    assert lib.dipsd_spec_verify(2, pa, pu, 7, 100, 0, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, 1 << 20,
                                  None) == 1
     a, pa = _i32([2, 3])
-    assert lib.dipsd_spec_verify(2, pa, 0, 0, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, 1 << 20,
+    assert lib.dipsd_spec_verify(2, pa, pu, 7, 0, 0, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, 1 << 20,
                                  None) == 1
-    assert lib.dipsd_spec_verify(2, pa, 100, 7, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, 1 << 20,
+    assert lib.dipsd_spec_verify(2, pa, pu, 7, 100, 7, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, 1 << 20,
                                  None) == 1
-    assert lib.dipsd_spec_verify(2, pa, 100, 0, FAKE, None, FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, 1 << 20,
+    assert lib.dipsd_spec_verify(2, pa, pu, 7, 100, 0, FAKE, None, FAKE, FAKE, FAKE, FAKE, None, FAKE, 1 << 20,
+                                 None) == 1
+    # user ids: required, non-negative
+    assert lib.dipsd_spec_verify(2, pa, None, 7, 100, 0, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, 1 << 20,
+                                 None) == 1
+    bad, pbad = _i32([0, -4])
+    assert lib.dipsd_spec_verify(2, pa, pbad, 7, 100, 0, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, 1 << 20,
                                  None) == 1
     # workspace too small / missing
-    assert lib.dipsd_spec_verify(2, pa, 100, 0, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, 8,
+    assert lib.dipsd_spec_verify(2, pa, pu, 7, 100, 0, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, 8,
                                  None) == 4
-    assert lib.dipsd_spec_verify(2, pa, 100, 0, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None, None, 1 << 20,
+    assert lib.dipsd_spec_verify(2, pa, pu, 7, 100, 0, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None, None, 1 << 20,
                                  None) == 4
+
+
+def test_noalloc_rejects_batches_beyond_its_positions_before_any_launch(lib):
+    a, pa = _i32([31] * 128 + [0])  # 4097 verify positions > DIPSD_NOALLOC_MAX_POSITIONS
+    u, pu = _i32(range(129))
+    n0 = lib.dipsd_launch_count()
+    assert lib.dipsd_spec_verify_noalloc(129, pa, pu, 3, 1024, 0, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None,
+                                         None) == 2
+    assert lib.dipsd_launch_count() == n0
+
+
+def test_philox_entry_points_reject_bad_arguments(lib):
+    assert lib.dipsd_philox_words(1, -1, 4, FAKE, None) == 1
+    assert lib.dipsd_philox_words(1, 0, -4, FAKE, None) == 1
+    assert lib.dipsd_philox_words(1, 0, 4, FAKE + 8, None) == 1  # not 16-byte aligned
+    assert lib.dipsd_philox_words(1, 0, 0, None, None) == 0      # nothing to write
+    a, pa = _i32([2, 3])
+    u, pu = _i32([0, -1])
+    assert lib.dipsd_verify_uniforms(2, pa, pu, 5, FAKE, None) == 1
+    u, pu = _i32([0, 1])
+    assert lib.dipsd_verify_uniforms(2, pa, pu, 5, None, None) == 1
+
+
+def test_test_overrides_are_explicit(lib):
+    """The planner never reads the environment: only dipsd_test_set_override moves it."""
+    import os
+    from paper_2604_20919_gb300 import dipsd
+    L, ctx = [5, 0, 8, 2, 20, 1], [1500, 3000, 333, 64, 700, 0]
+    base = dipsd.dipsd_verify_attention_plan(L, ctx, 64, 8, 128, 152)
+    os.environ["DIPSD_ATTN_CLUSTER"] = "3"
+    try:
+        assert dipsd.dipsd_verify_attention_plan(L, ctx, 64, 8, 128, 152)["cluster"] == base["cluster"]
+    finally:
+        del os.environ["DIPSD_ATTN_CLUSTER"]
+    with dipsd.plan_override(attn_cluster=3):
+        assert dipsd.dipsd_verify_attention_plan(L, ctx, 64, 8, 128, 152)["cluster"] == 3
+    assert dipsd.dipsd_verify_attention_plan(L, ctx, 64, 8, 128, 152)["cluster"] == base["cluster"]
+    assert lib.dipsd_test_set_override(0, 1) == 1
+    assert lib.dipsd_test_set_override(7, 1) == 1
+    assert lib.dipsd_test_set_override(1, -1) == 1
 
 
 def test_spec_workspace_size_is_host_only(lib):
@@ -104,7 +151,7 @@ def test_verify_batch_rejects_bad_membership(lib):
     m, pm = _i32([0, 2, 2])
     a, pa = _i32([1, 2, 3])
     c, pc = _i32([4, 4, 4])
-    args = (FAKE, FAKE, FAKE, 16, FAKE, 4, 8, 2, 128, 0.1, FAKE + 4096, 100, 0, FAKE, FAKE, FAKE, FAKE,
+    args = (FAKE, FAKE, FAKE, 16, FAKE, 4, 8, 2, 128, 0.1, FAKE + 4096, 100, 0, FAKE, FAKE, FAKE, 7,
             FAKE, FAKE, FAKE, None, FAKE, 1 << 20, None)
     assert lib.dipsd_verify_batch(3, pm, 3, pa, pc, *args) == 1   # duplicate member
     m, pm = _i32([0, 3])

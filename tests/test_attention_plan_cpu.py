@@ -3,7 +3,6 @@ dipsd_verify_attention_plan: every key of every user is covered by its KV
 splits, the work-item count and the grid follow from them, and the persistent
 grid, the cluster merge and the merge kernel are chosen only where the kernel
 supports them."""
-import os
 
 import numpy as np
 import pytest
@@ -20,24 +19,6 @@ def dipsd():
     build.build()
     d.load()
     return d
-
-
-class _env:
-    """Sets DIPSD_* planner overrides for the duration of a block."""
-
-    def __init__(self, **kv):
-        self.kv = {k: str(v) for k, v in kv.items()}
-
-    def __enter__(self):
-        self.old = {k: os.environ.get(k) for k in self.kv}
-        os.environ.update(self.kv)
-
-    def __exit__(self, *exc):
-        for k, v in self.old.items():
-            if v is None:
-                del os.environ[k]
-            else:
-                os.environ[k] = v
 
 
 def _check_plan(p, L, ctx, Hq, Hkv, D, num_sms, append, forced_cluster=False):
@@ -113,17 +94,17 @@ def test_plan_of_the_workloads(dipsd):
 
 def test_plan_overrides(dipsd):
     L, ctx = [5, 0, 8, 2, 20, 1], [1500, 3000, 333, 64, 700, 0]
-    with _env(DIPSD_ATTN_PERSIST=1, DIPSD_ATTN_GRID=7, DIPSD_ATTN_SPLIT_TILES=2):
+    with dipsd.plan_override(attn_persist=1, attn_grid=7, attn_split_tiles=2):
         p = dipsd.dipsd_verify_attention_plan(L, ctx, 64, 8, 128, 152)
         assert p["grid"] == 7 and p["n_items"] > 7 and p["n_merge"] > 0
         _check_plan(p, L, ctx, 64, 8, 128, 152, False)
         pa = dipsd.dipsd_verify_attention_plan(L, ctx, 64, 8, 128, 152, append=True)
         assert pa["grid"] == pa["n_items"]  # the append keeps one item per CTA
-    with _env(DIPSD_ATTN_PERSIST=0):
+    with dipsd.plan_override(attn_persist=2):
         s = config_shape(3, 0)
         p = dipsd.dipsd_verify_attention_plan(s["L"], s["ctx"], s["Hq"], s["Hkv"], s["D"], 152)
         assert p["grid"] == p["n_items"]
-    with _env(DIPSD_ATTN_CLUSTER=3):
+    with dipsd.plan_override(attn_cluster=3):
         p = dipsd.dipsd_verify_attention_plan(L, ctx, 64, 8, 128, 152)
         assert p["cluster"] == 3 and (p["nsplit"] == 3).all()
         _check_plan(p, L, ctx, 64, 8, 128, 152, False, forced_cluster=True)

@@ -5,7 +5,6 @@ slots are poisoned with NaN, and the append entry point gets the rows as
 inputs: its attention must match the oracle on the untouched cache, and the
 cache must come back bit for bit (oracle.kv_append on the poisoned cache
 gives the same bytes)."""
-import os
 
 import numpy as np
 import pytest
@@ -72,21 +71,13 @@ def test_append_attention_edges(cuda_lib, L, ctx, Hq, Hkv, D):
     check_attention(_append_run(cuda_lib, b), _reference(b))
 
 
-@pytest.mark.parametrize("env,val", [("DIPSD_ATTN_SPLIT_TILES", "1"), ("DIPSD_ATTN_SPLIT_TILES", "3"),
-                                     ("DIPSD_ATTN_CLUSTER", "3"),
-                                     ("DIPSD_ATTN_PERSIST", "1")])
-def test_append_with_splits(cuda_lib, env, val):
+@pytest.mark.parametrize("override,val", [("attn_split_tiles", 1), ("attn_split_tiles", 3), ("attn_cluster", 3),
+                                          ("attn_persist", 1)])
+def test_append_with_splits(cuda_lib, override, val):
     """Splits of one tile each put the new rows of a user into two CTAs."""
     b = make_batch([31, 5, 0, 12], [50, 1000, 63, 200], Hq=64, Hkv=8, D=128, V=64, seed=47)
-    old = os.environ.get(env)
-    os.environ[env] = val
-    try:
+    with cuda_lib.plan_override(**{override: val}):
         out = _append_run(cuda_lib, b)
-    finally:
-        if old is None:
-            del os.environ[env]
-        else:
-            os.environ[env] = old
     check_attention(out, _reference(b))
 
 
@@ -96,11 +87,12 @@ def test_batch_append_matches_batch(cuda_lib):
     nk, nv, kc, vc = _split_new_rows(b)
     g = lambda t: t.to(DEV)
     q, bt = g(b.q), g(b.block_table)
-    z, w, d, u = g(b.target_logits), g(b.draft_logits), g(b.draft_tokens), g(b.uniforms)
-    ref = cuda_lib.dipsd_verify_batch(b.members, b.L, b.ctx, q, g(b.k_cache), g(b.v_cache), bt, b.scale, z, w, d, u)
+    z, w, d = g(b.target_logits), g(b.draft_logits), g(b.draft_tokens)
+    ref = cuda_lib.dipsd_verify_batch(b.members, b.L, b.ctx, q, g(b.k_cache), g(b.v_cache), bt, b.scale, z, w, d,
+                                      b.seed)
     kc_d, vc_d = g(kc), g(vc)
     res = cuda_lib.dipsd_verify_batch_append(b.members, b.L, b.ctx, q, g(nk), g(nv), kc_d, vc_d, bt, b.scale,
-                                             z, w, d, u)
+                                             z, w, d, b.seed)
     torch.cuda.synchronize()
     assert torch.equal(res[0], ref[0])
     for x, y in zip(valid_spec_outputs(*res[1:]), valid_spec_outputs(*ref[1:])):

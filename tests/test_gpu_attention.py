@@ -1,5 +1,4 @@
 """verify_attention through the C ABI vs the fp64 oracle."""
-import os
 
 import pytest
 import torch
@@ -59,42 +58,27 @@ def test_attention_edge_shapes(cuda_lib, L, ctx, Hq, Hkv, D):
     check_attention(_run(cuda_lib, b), _full_reference(b))
 
 
-@pytest.mark.parametrize("split_tiles", ["1", "2", "7"])
+@pytest.mark.parametrize("split_tiles", [1, 2, 7])
 def test_attention_forced_splits(cuda_lib, split_tiles):
     """Many KV splits per (user, head) exercise the partial/merge path."""
     b = make_batch([5, 0, 8, 2], [1500, 3000, 333, 64], Hq=64, Hkv=8, D=128, V=64, seed=21)
-    old = os.environ.get("DIPSD_ATTN_SPLIT_TILES")
-    os.environ["DIPSD_ATTN_SPLIT_TILES"] = split_tiles
-    try:
+    with cuda_lib.plan_override(attn_split_tiles=split_tiles):
         out = _run(cuda_lib, b)
-    finally:
-        if old is None:
-            del os.environ["DIPSD_ATTN_SPLIT_TILES"]
-        else:
-            os.environ["DIPSD_ATTN_SPLIT_TILES"] = old
     check_attention(out, _full_reference(b))
 
 
-@pytest.mark.parametrize("cluster,D", [("2", 128), ("3", 128), ("6", 64)])
+@pytest.mark.parametrize("cluster,D", [(2, 128), (3, 128), (6, 64)])
 def test_attention_cluster_merge(cuda_lib, cluster, D):
     """KV splits merged inside a thread-block cluster, including empty splits
     (a user with fewer 64-key tiles than splits)."""
     b = make_batch([5, 0, 8, 2, 1], [1500, 3000, 333, 64, 0], Hq=64 if D == 128 else 16, Hkv=8 if D == 128 else 2,
                    D=D, V=64, seed=23)
-    old = os.environ.get("DIPSD_ATTN_CLUSTER")
-    os.environ["DIPSD_ATTN_CLUSTER"] = cluster
-    try:
+    with cuda_lib.plan_override(attn_cluster=cluster):
         out = _run(cuda_lib, b)
-    finally:
-        if old is None:
-            del os.environ["DIPSD_ATTN_CLUSTER"]
-        else:
-            os.environ["DIPSD_ATTN_CLUSTER"] = old
     check_attention(out, _full_reference(b))
 
 
-@pytest.mark.parametrize("grid,split_tiles,D", [("1", None, 128), ("3", None, 128), ("7", "2", 128),
-                                                 ("5", "1", 64), ("152", "1", 128)])
+@pytest.mark.parametrize("grid,split_tiles,D", [(1, 0, 128), (3, 0, 128), (7, 2, 128), (5, 1, 64), (152, 1, 128)])
 def test_attention_persistent_grid(cuda_lib, grid, split_tiles, D):
     """A grid smaller than the item count: each CTA walks several items (row
     blocks with and without padding rows, ragged last tiles, KV splits and
@@ -102,21 +86,10 @@ def test_attention_persistent_grid(cuda_lib, grid, split_tiles, D):
     items."""
     b = make_batch([5, 0, 8, 2, 20, 1], [1500, 3000, 333, 64, 700, 0], Hq=64 if D == 128 else 16,
                    Hkv=8 if D == 128 else 2, D=D, V=64, seed=24)
-    env = {"DIPSD_ATTN_PERSIST": "1", "DIPSD_ATTN_GRID": grid}
-    if split_tiles:
-        env["DIPSD_ATTN_SPLIT_TILES"] = split_tiles
-    old = {k: os.environ.get(k) for k in env}
-    os.environ.update(env)
-    try:
+    with cuda_lib.plan_override(attn_persist=1, attn_grid=grid, attn_split_tiles=split_tiles):
         ws = cuda_lib.workspace(cuda_lib.dipsd_verify_attention_workspace_size(b.L, b.ctx, b.Hq, b.Hkv, b.D), DEV)
         out = _run(cuda_lib, b, ws)
         assert cuda_lib.device_status(ws) == 0
-    finally:
-        for k, v in old.items():
-            if v is None:
-                del os.environ[k]
-            else:
-                os.environ[k] = v
     check_attention(out, _full_reference(b))
 
 

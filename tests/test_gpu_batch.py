@@ -6,7 +6,7 @@ import torch
 
 import oracle
 from parity import attention_subset_reference, check_attention, check_spec, valid_spec_outputs
-from workloads import make_config
+from workloads import make_batch, make_config
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda"
@@ -17,7 +17,7 @@ def _launch(dipsd, b, L_all, ctx_all, kc, vc, bt, stream):
     with torch.cuda.stream(stream):
         res = dipsd.dipsd_verify_batch(b.members, L_all, ctx_all, g(b.q), kc, vc, bt, b.scale,
                                        g(b.target_logits), g(b.draft_logits), g(b.draft_tokens),
-                                       g(b.uniforms), stream=stream)
+                                       b.seed, stream=stream)
     return res
 
 
@@ -44,10 +44,10 @@ def test_batch_matches_separate_calls(cuda_lib):
     b = make_config(2, seed=4)
     g = lambda t: t.to(DEV)
     q, kc, vc, bt = g(b.q), g(b.k_cache), g(b.v_cache), g(b.block_table)
-    z, w, d, u = g(b.target_logits), g(b.draft_logits), g(b.draft_tokens), g(b.uniforms)
+    z, w, d = g(b.target_logits), g(b.draft_logits), g(b.draft_tokens)
     attn_a = cuda_lib.dipsd_verify_attention(b.L, b.ctx, q, kc, vc, bt, b.scale)
-    sv = cuda_lib.dipsd_spec_verify(b.L, z, w, d, u)
-    res = cuda_lib.dipsd_verify_batch(b.members, b.L, b.ctx, q, kc, vc, bt, b.scale, z, w, d, u)
+    sv = cuda_lib.dipsd_spec_verify(b.L, b.members, b.seed, z, w, d)
+    res = cuda_lib.dipsd_verify_batch(b.members, b.L, b.ctx, q, kc, vc, bt, b.scale, z, w, d, b.seed)
     torch.cuda.synchronize()
     assert torch.equal(attn_a, res[0])
     for x, y in zip(valid_spec_outputs(*sv), valid_spec_outputs(*res[1:])):
@@ -56,9 +56,12 @@ def test_batch_matches_separate_calls(cuda_lib):
 
 def test_batch_with_permuted_membership(cuda_lib):
     """Members name rows of a larger user table, in any order."""
-    b = make_config(1, seed=5)
-    # table of 6 users: batch users sit at rows 4, 0, 5, 2
+    # table of 6 users: batch users sit at rows 4, 0, 5, 2 (their Philox key words)
     perm = np.array([4, 0, 5, 2])
+    from workloads import config_shape
+    s = config_shape(1)
+    b = make_batch(s["L"], s["ctx"], Hq=s["Hq"], Hkv=s["Hkv"], D=s["D"], V=s["V"], logit_std=s["logit_std"],
+                   noise_sigma=s["noise_sigma"], logit_dtype=s["logit_dtype"], seed=5, user_ids=perm)
     L_all = np.zeros(6, np.int32)
     ctx_all = np.zeros(6, np.int32)
     L_all[perm], ctx_all[perm] = b.L, b.ctx
@@ -67,7 +70,7 @@ def test_batch_with_permuted_membership(cuda_lib):
     g = lambda t: t.to(DEV)
     attn, acc, offs, toks, probs = cuda_lib.dipsd_verify_batch(
         perm, L_all, ctx_all, g(b.q), g(b.k_cache), g(b.v_cache), g(bt_all), b.scale, g(b.target_logits),
-        g(b.draft_logits), g(b.draft_tokens), g(b.uniforms))
+        g(b.draft_logits), g(b.draft_tokens), b.seed)
     torch.cuda.synchronize()
     ref = oracle.verify_attention(b.q.double().numpy(), b.k_cache.double().numpy(), b.v_cache.double().numpy(),
                                   b.block_table.numpy(), b.ctx, b.L, b.scale)

@@ -17,8 +17,8 @@ DEV = "cuda"
 
 def _run(dipsd, b, sd, ws=None):
     g = lambda t: t.to(DEV)
-    res = dipsd.dipsd_spec_verify_sparse(b.L, g(b.target_logits), g(sd.draft_tokens), g(sd.draft_logq),
-                                         g(sd.topk_idx), g(sd.topk_q), g(b.uniforms), ws=ws)
+    res = dipsd.dipsd_spec_verify_sparse(b.L, b.user_ids, b.seed, g(b.target_logits), g(sd.draft_tokens),
+                                         g(sd.draft_logq), g(sd.topk_idx), g(sd.topk_q), ws=ws)
     torch.cuda.synchronize()
     return res
 

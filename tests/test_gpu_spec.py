@@ -15,8 +15,8 @@ DEV = "cuda"
 
 def _run(dipsd, b, stream=None):
     g = lambda t: t.to(DEV)
-    out = dipsd.dipsd_spec_verify(b.L, g(b.target_logits), g(b.draft_logits), g(b.draft_tokens),
-                                  g(b.uniforms), stream=stream)
+    out = dipsd.dipsd_spec_verify(b.L, b.user_ids, b.seed, g(b.target_logits), g(b.draft_logits),
+                                  g(b.draft_tokens), stream=stream)
     torch.cuda.synchronize()
     return out
 
@@ -132,11 +132,9 @@ def test_spec_verify_output_law_monte_carlo(cuda_lib):
     acc_hits = np.zeros(L)
     for c in range(calls):
         d = np.stack([rng.choice(V, size=users, p=q[t]) for t in range(L)], axis=1).reshape(-1)
-        u = rng.random((users * (L + 1), 2)).astype(np.float32)
-        u = np.clip(u, 1e-7, 1 - 1e-7)
+        # a fresh seed per call: the in-kernel Philox uniforms are the only randomness
         acc, offs, toks, _ = cuda_lib.dipsd_spec_verify(
-            [L] * users, z, w, torch.tensor(d, dtype=torch.int32, device=DEV),
-            torch.tensor(u, device=DEV))
+            [L] * users, np.arange(users), 1000 + c, z, w, torch.tensor(d, dtype=torch.int32, device=DEV))
         a = acc.cpu().numpy()
         o = offs.cpu().numpy()
         tk = toks.cpu().numpy()

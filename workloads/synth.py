@@ -26,9 +26,11 @@ Recipe (seeded, reproducible):
   * draft tokens d ~ softmax(w_stored), drawn with the Gumbel-max trick in
     fp64 from a seeded numpy stream (the drafting device's job, Sec. II-A
     step 1; not the verifier's arithmetic).
-  * uniforms: two per verify position (acceptance, resample) from a Philox
-    counter-based stream keyed on (seed, user id), position-indexed, mapped
-    to (k + 0.5) * 2^-23 so every value is an exact fp32 in (0, 1).
+  * uniforms: two per verify position (acceptance, resample) from numpy's
+    Philox4x64-10 stream keyed on (seed, user id): position t takes words 2t
+    and 2t + 1, each mapped to ((w >> 41) + 0.5) * 2^-23, an exact fp32 in
+    (0, 1).  The CUDA library draws the same words with its own Philox; the
+    oracle reads these host copies.
 """
 from __future__ import annotations
 
@@ -106,9 +108,10 @@ class Batch:
     target_logits: torch.Tensor  # [sum T, V]
     draft_logits: torch.Tensor   # [sum L, V]
     draft_tokens: torch.Tensor   # int32 [sum L]
-    uniforms: torch.Tensor       # fp32 [sum T, 2]: (u_accept, u_resample)
+    uniforms: torch.Tensor       # fp32 [sum T, 2]: (u_accept, u_resample), host, for the oracle
     alpha: np.ndarray = field(default=None)  # design acceptance per user
-    seed: int = 0
+    seed: int = 0                # Philox key word 0
+    user_ids: np.ndarray = field(default=None)  # int32 [B]: Philox key word 1 per batch user
 
     @property
     def B(self) -> int:
@@ -254,8 +257,8 @@ def make_batch(L, ctx, *, Hq, Hkv, D, V, logit_std=1.0, noise_sigma=1.0,
                  logit_dtype=logit_dtype, q=q, k_cache=k_cache, v_cache=v_cache,
                  block_table=torch.from_numpy(bt).to(device),
                  target_logits=zt.to(device), draft_logits=wt.to(device),
-                 draft_tokens=d.to(device), uniforms=uni.to(device),
-                 alpha=None if alpha is None else np.asarray(alpha, np.float64), seed=seed)
+                 draft_tokens=d.to(device), uniforms=uni,
+                 alpha=None if alpha is None else np.asarray(alpha, np.float64), seed=seed, user_ids=uid)
 
 
 # ----------------------------------------------------------------------------
@@ -344,6 +347,6 @@ def make_pipeline(s, seed, device, kv_device):
                              V=s["V"], logit_dtype=s["logit_dtype"], q=q.to(device),
                              k_cache=k_cache, v_cache=v_cache, block_table=bt_t,
                              target_logits=zt.to(device), draft_logits=wt.to(device),
-                             draft_tokens=d.to(device), uniforms=uni.to(device),
-                             alpha=alpha[mem], seed=seed))
+                             draft_tokens=d.to(device), uniforms=uni,
+                             alpha=alpha[mem], seed=seed, user_ids=mem.astype(np.int32)))
     return batches
