@@ -7,11 +7,18 @@ speculative sampling over the vocabulary) on the Qwen3-32B-shaped batch
 (B=8, L_i ~ U{1..8}, context 1024, 64/8/128 heads, V=151936).  Inputs are
 resident in HBM; consecutive steps rotate over enough device copies of the
 batch that their inputs exceed L2, so every step reads cold data; the K calls
-are captured in one CUDA graph and run back to back as one replay between a
-pair of CUDA events.  The line also carries the end-to-end number through the
-same call with host buffers (copies inside the timed region), per-stage
-roofline figures against the measured HBM copy bandwidth, the clocks seen
-while timing, and the fp64 CPU oracle timed on the host cores.
+are captured in one CUDA graph, and the graph is replayed back to back until
+at least --min-replay-ms of device time has run, each replay of exactly K
+steps between a pair of CUDA events: the value is the median replay, with the
+spread beside it.  The line also carries:
+  * e2e: the same steps through the Python API as plain calls (the library's
+    host validation and planning included), each step copying its inputs from
+    pinned host memory and its results back; e2e_graph: the same calls
+    captured as one CUDA graph;
+  * per-stage roofline figures against the measured HBM copy bandwidth, on
+    this workload and (--extra 1, the default) on workloads 3 and 4, and the
+    sustained rate of workload 5's pipelined schedule;
+  * the clocks seen while timing, and the fp64 CPU oracle on the host cores.
 
 Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl dipsd|reference]
 Under torchrun (N > 1) every rank verifies its own replica of the batch.
@@ -46,6 +53,10 @@ def parse_args():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--cpu-seconds", type=float, default=10.0,
                     help="budget of the CPU oracle baseline (0: skip it, for the large non-headline workloads)")
+    ap.add_argument("--min-replay-ms", type=float, default=300.0,
+                    help="device time each timed graph is replayed for (at least 3 replays)")
+    ap.add_argument("--extra", type=int, default=1,
+                    help="1: also time workloads 3 and 4 per stage and workload 5's pipelined schedule")
     return ap.parse_args()
 
 
@@ -54,6 +65,26 @@ def workload_config(b, wl, seed):
     return {"workload": CONFIG_NAMES[wl], "B": int(b.B), "L": [int(x) for x in b.L],
             "ctx": [int(x) for x in b.ctx], "heads": f"{b.Hq}/{b.Hkv}/{b.D}", "V": int(b.V),
             "page": 16, "seed": seed}
+
+
+def step_bytes(b):
+    return attention_bytes(b) + spec_bytes(b)
+
+
+def copies_for(b):
+    """Device copies of a batch that consecutive steps rotate over: their
+    inputs together exceed L2 twice over, so every step reads cold data."""
+    return max(2, math.ceil(2 * L2_BYTES / step_bytes(b)))
+
+
+def bench_config(b, wl, seed, world):
+    """`config` of the bench line, the same in both arms."""
+    cfg = workload_config(b, wl, seed)
+    R = copies_for(b)
+    cfg["l2"] = (f"inputs rotated over {R} device copies ({R * step_bytes(b) / 1e6:.0f} MB > 2 x L2), "
+                 "K steps back to back as one CUDA graph replay")
+    cfg["parallelism"] = "replicas" if world > 1 else "single"
+    return cfg
 
 
 def read_peaks():
@@ -200,9 +231,9 @@ def cpu_baseline(b, budget_s):
 
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
     if rank != 0:
         return
-    import torch
     from workloads import make_config
     b = make_config(args.workload, seed=args.seed, device="cpu")
     hb = host_copy(b)
@@ -219,12 +250,127 @@ def run_reference(args):
             "value": value, "unit": "verified tokens/s", "n_gpus": args.gpus, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": 1000 * dt / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": workload_config(b, args.workload, args.seed), "impl": "reference",
+            "config": bench_config(b, args.workload, args.seed, world), "impl": "reference",
             "cpu_baseline": {"value": value, "unit": "verified tokens/s", "cores": os.cpu_count(),
                              "kind": "oracle", "sample": f"{args.steps} full batch(es) of the workload"},
             "e2e": {"value": value, "unit": "verified tokens/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------- timing
+def capture(fn, n, R, stream):
+    """A CUDA graph of n consecutive calls fn(0), .., fn(n - 1) (lazy set-up
+    settled outside the capture) and the library kernels one replay launches."""
+    import torch
+    from paper_2604_20919_gb300 import dipsd
+    g = torch.cuda.CUDAGraph()
+    side = torch.cuda.Stream()
+    side.wait_stream(stream)
+    with torch.cuda.stream(side):
+        for i in range(R):
+            fn(i)
+    stream.wait_stream(side)
+    torch.cuda.synchronize()
+    n0 = dipsd.dipsd_launch_count()
+    with torch.cuda.graph(g):
+        for i in range(n):
+            fn(i)
+    torch.cuda.synchronize()
+    return g, dipsd.dipsd_launch_count() - n0
+
+
+def replay_ms(g, stream, reps, barrier=None):
+    """reps replays of a graph, each between a pair of CUDA events on the
+    launching stream (synchronised on both sides): ms per replay."""
+    import torch
+    out = []
+    for _ in range(reps):
+        if barrier:
+            barrier()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        g.replay()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        out.append(e0.elapsed_time(e1))
+    return out
+
+
+def replay_stats(g, n, stream, min_ms):
+    """ms per call of an n-call graph: median, min and max over replays run
+    until min_ms of device time (at least 3 replays)."""
+    first = replay_ms(g, stream, 2)[1]
+    reps = max(3, min(2000, math.ceil(min_ms / max(first, 1e-3))))
+    t = np.asarray(replay_ms(g, stream, reps)) / n
+    return {"ms": float(np.median(t)), "ms_min": float(t.min()), "ms_max": float(t.max()), "replays": reps,
+            "calls_per_replay": n}
+
+
+def stage_entry(st, alg_bytes, hbm_peak):
+    gbs = alg_bytes / st["ms"] / 1e6
+    return dict(st, alg_bytes=alg_bytes, gbs=gbs, frac_of_measured_hbm=gbs / hbm_peak, frac_of_8000=gbs / 8000.0)
+
+
+def device_batch(b, dev, R):
+    """R device copies of a batch's per-step inputs (the KV cache cloned too)."""
+    copies = []
+    for k in range(R):
+        kc = b.k_cache if k == 0 else b.k_cache.clone()
+        vc = b.v_cache if k == 0 else b.v_cache.clone()
+        copies.append(dict(q=b.q.to(dev), z=b.target_logits.to(dev), w=b.draft_logits.to(dev),
+                           d=b.draft_tokens.to(dev), kc=kc, vc=vc))
+    return copies
+
+
+def measure_workload(wl, args, dev, stream, hbm_peak):
+    """Per-stage times of one workload (attention alone, speculative sampling
+    alone, the whole verify_batch step), inputs rotated over device copies
+    larger than L2 twice over."""
+    import torch
+    from paper_2604_20919_gb300 import dipsd
+    from workloads import CONFIG_NAMES, make_config
+    b = make_config(wl, seed=args.seed, device="cpu", kv_device=dev)
+    R = copies_for(b)
+    copies = device_batch(b, dev, R)
+    bt = b.block_table.to(dev)
+    attn_out = torch.empty_like(copies[0]["q"])
+    outs = dipsd.spec_outputs(b.L, dev)
+    ws = dipsd.workspace(dipsd.dipsd_verify_batch_workspace_size(b.members, b.L, b.ctx, b.Hq, b.Hkv, b.D, b.V), dev)
+
+    def step(k):
+        c = copies[k % R]
+        dipsd.dipsd_verify_batch(b.members, b.L, b.ctx, c["q"], c["kc"], c["vc"], bt, b.scale, c["z"], c["w"],
+                                 c["d"], b.seed, attn_out=attn_out, outputs=outs, ws=ws)
+
+    def attn_only(k):
+        c = copies[k % R]
+        dipsd.dipsd_verify_attention(b.L, b.ctx, c["q"], c["kc"], c["vc"], bt, b.scale, out=attn_out, ws=ws)
+
+    def spec_only(k):
+        c = copies[k % R]
+        dipsd.dipsd_spec_verify(b.L, b.members, b.seed, c["z"], c["w"], c["d"], outputs=outs, ws=ws)
+
+    for i in range(3):
+        step(i)
+    torch.cuda.synchronize()
+    # about 20 ms of device time per replay
+    n = int(min(500, max(5, 0.02 / (step_bytes(b) / 4.0e12))))
+    res = {"workload": CONFIG_NAMES[wl], "B": int(b.B), "sum_T": int(b.sum_T)}
+    for name, fn, by in (("step", step, step_bytes(b)), ("verify_attention", attn_only, attention_bytes(b)),
+                         ("spec_verify", spec_only, spec_bytes(b))):
+        g, _ = capture(fn, n, R, stream)
+        res[name] = stage_entry(replay_stats(g, n, stream, args.min_replay_ms), by, hbm_peak)
+        del g
+    emitted = int(outs[1][-1].item())
+    res["step"]["verified_tokens_per_s"] = emitted / (res["step"]["ms"] / 1000.0)
+    res["emitted_tokens_per_step"] = emitted
+    res["l2"] = f"inputs rotated over {R} device copies ({R * step_bytes(b) / 1e6:.0f} MB)"
+    assert dipsd.device_status(ws) == 0
+    del copies, attn_out, outs, ws, bt
+    torch.cuda.empty_cache()
+    return res
 
 
 def run_dipsd(args):
@@ -240,21 +386,14 @@ def run_dipsd(args):
     dev = torch.device("cuda", local)
     if world > 1:
         dist.init_process_group("nccl", device_id=dev)
+    barrier = dist.barrier if world > 1 else None
     dipsd.load()
+    hbm_peak, peak_kind = read_peaks()
 
     # each rank verifies its own replica (independent users): weak scaling, no collective
     b = make_config(args.workload, seed=args.seed + rank, device="cpu", kv_device=dev)
-    step_bytes = attention_bytes(b) + spec_bytes(b)
-    # R device-resident copies of the batch, used in rotation, so that the
-    # inputs of consecutive steps together exceed L2 twice over: every step
-    # reads cold data without a flush kernel between steps
-    R = max(2, math.ceil(2 * L2_BYTES / step_bytes))
-    copies = []
-    for k in range(R):
-        kc = b.k_cache if k == 0 else b.k_cache.clone()
-        vc = b.v_cache if k == 0 else b.v_cache.clone()
-        copies.append(dict(q=b.q.to(dev), z=b.target_logits.to(dev), w=b.draft_logits.to(dev),
-                           d=b.draft_tokens.to(dev), kc=kc, vc=vc))
+    R = copies_for(b)
+    copies = device_batch(b, dev, R)
     bt = b.block_table.to(dev)
     attn_out = torch.empty_like(copies[0]["q"])
     outs = dipsd.spec_outputs(b.L, dev)
@@ -300,40 +439,6 @@ def run_dipsd(args):
         dipsd.dipsd_verify_attention_append(b.L, b.ctx, c["q"], new_k, new_v, c["kc"], c["vc"], bt, b.scale,
                                             out=attn_out, ws=ws)
 
-    def graph_of(fn, n):
-        """A CUDA graph of n consecutive calls cycling over the R input copies,
-        and the number of library kernels it launches per replay."""
-        g = torch.cuda.CUDAGraph()
-        side = torch.cuda.Stream()
-        side.wait_stream(stream)
-        with torch.cuda.stream(side):
-            for i in range(R):  # settle lazy set-up outside the capture
-                fn(i)
-        stream.wait_stream(side)
-        torch.cuda.synchronize()
-        n0 = dipsd.dipsd_launch_count()
-        with torch.cuda.graph(g):
-            for i in range(n):
-                fn(i)
-        torch.cuda.synchronize()
-        return g, dipsd.dipsd_launch_count() - n0
-
-    def timed(g, n):
-        """One replay (n calls back to back) between a pair of CUDA events, after a
-        warm replay; returns ms per call."""
-        g.replay()
-        if world > 1:
-            dist.barrier()
-        torch.cuda.synchronize()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        g.replay()
-        e1.record(stream)
-        torch.cuda.synchronize()
-        if world > 1:
-            dist.barrier()
-        return e0.elapsed_time(e1) / n
-
     def cold_latency(fn, k):
         """Single calls with L2 flushed (a 256 MB write) before each, outside the events."""
         evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(k)]
@@ -353,26 +458,33 @@ def run_dipsd(args):
     assert dipsd.device_status(ws) == 0
 
     n_steps = args.steps
-    g_step, launches = graph_of(step, n_steps)
-    g_attn, _ = graph_of(attn_only, n_steps)
-    g_spec, _ = graph_of(spec_only, n_steps)
-    g_app, _ = graph_of(attn_append, n_steps)
-    g_sps, _ = graph_of(spec_sparse, n_steps)
+    g_step, launches = capture(step, n_steps, R, stream)
 
     sampler = ClockSampler(local)
     sampler.start()
-    ms_step = timed(g_step, n_steps)
-    ms_attn = timed(g_attn, n_steps)
-    ms_spec = timed(g_spec, n_steps)
-    ms_app = timed(g_app, n_steps)
-    ms_sps = timed(g_sps, n_steps)
+    # the headline: replays of exactly K steps, as many on every rank (the
+    # count agreed before timing), median over the replays
+    first = replay_ms(g_step, stream, 2, barrier)[1]
+    reps = max(3, min(2000, math.ceil(args.min_replay_ms / max(first, 1e-3))))
+    if world > 1:
+        t = torch.tensor([reps], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        reps = int(t.item())
+    step_ms = np.asarray(replay_ms(g_step, stream, reps, barrier))
+    total_ms = float(np.median(step_ms))
+
+    stages = {}
+    for name, fn in (("verify_attention", attn_only), ("spec_verify", spec_only),
+                     ("verify_attention_append", attn_append), ("spec_verify_sparse", spec_sparse)):
+        g, _ = capture(fn, n_steps, R, stream)
+        stages[name] = replay_stats(g, n_steps, stream, args.min_replay_ms / 3)
+        del g
     lat_step = cold_latency(step, min(args.steps, 50))
 
-    # end to end through the same call: every step copies its inputs from pinned
-    # host memory into one of the R device copies (copy stream), runs the call,
-    # and reads its results back into per-copy pinned buffers (compute stream);
-    # step k+1's upload overlaps step k's compute.  R steps are captured as one
-    # graph, replayed back to back, timed on the host clock.
+    # end to end through the Python API: every step copies its inputs from
+    # pinned host memory into one of the R device copies (copy stream), makes
+    # the call and reads its results back into per-copy pinned buffers
+    # (compute stream); step k+1's upload overlaps step k's compute.
     pin = lambda t: t.cpu().pin_memory()
     keys = ("q", "z", "w", "d")
     h_in = [pin(x) for x in (b.q, b.target_logits, b.draft_logits, b.draft_tokens)]
@@ -380,8 +492,9 @@ def run_dipsd(args):
     h2d = sum(x.numel() * x.element_size() for x in h_in)
     d2h = sum(x.numel() * x.element_size() for x in h_out[0])
     cs = torch.cuda.Stream()
+    api_s = [0.0]
 
-    def e2e_steps(n):
+    def e2e_steps(n, host_clock=False):
         free = [None] * R
         cs.wait_stream(stream)
         for i in range(n):
@@ -395,65 +508,81 @@ def run_dipsd(args):
                 up = torch.cuda.Event()
                 up.record(cs)
             stream.wait_event(up)
+            t0 = time.perf_counter()
             step(k)
+            if host_clock:
+                api_s[0] += time.perf_counter() - t0
             for hd, dd in zip(h_out[k], outs[:3]):
                 hd.copy_(dd, non_blocking=True)
             free[k] = torch.cuda.Event()
             free[k].record(stream)
         stream.wait_stream(cs)
 
-    e2e_steps(R)  # settle outside the capture
+    # plain calls: the library's host work (validation, planning, launches)
+    # and the binding's argument marshalling are inside the timed region
+    e2e_steps(R)
     torch.cuda.synchronize()
+    if barrier:
+        barrier()
+    t0 = time.perf_counter()
+    e2e_steps(n_steps, host_clock=True)
+    torch.cuda.synchronize()
+    e2e_plain_ms = 1000 * (time.perf_counter() - t0) / n_steps
+    api_us = 1e6 * api_s[0] / n_steps
+    # the same steps captured as one CUDA graph, replayed back to back
     g_e2e = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g_e2e):
         e2e_steps(R)
     g_e2e.replay()
     torch.cuda.synchronize()
-    reps = max(1, args.steps // R)
+    reps_g = max(1, n_steps // R)
     t0 = time.perf_counter()
-    for _ in range(reps):
+    for _ in range(reps_g):
         g_e2e.replay()
     torch.cuda.synchronize()
-    e2e_ms = [1000 * (time.perf_counter() - t0) / (reps * R)] * args.steps
+    e2e_graph_ms = 1000 * (time.perf_counter() - t0) / (reps_g * R)
     clocks = sampler.stop()
 
     emitted = int(outs[1][-1].item())
     units = emitted * n_steps
-    total_ms = ms_step * n_steps
     from paper_2604_20919_gb300.shard import aggregate_timing
-    total_ms_max, units_all, e2e_max = aggregate_timing(total_ms, units, float(np.sum(e2e_ms)), device=dev)
+    total_ms_max, units_all, e2e_max = aggregate_timing(total_ms, units, e2e_plain_ms * n_steps, device=dev)
+    extra = {}
+    if args.extra and world == 1:
+        del g_step, g_e2e
+        del copies, new_k, new_v, flush
+        torch.cuda.empty_cache()
+        for wl in (3, 4):
+            if wl != args.workload:
+                extra[f"stages_workload{wl}"] = measure_workload(wl, args, dev, stream, hbm_peak)
+        extra["workload5"] = measure_pipeline(args, dev)
     if rank != 0:
         if world > 1:
             dist.destroy_process_group()
         return
+    write_line(args, b, world, hbm_peak, peak_kind, stages, total_ms_max, units_all, n_steps, step_ms, emitted,
+               launches, lat_step, e2e_max, e2e_graph_ms, api_us, h2d, d2h, clocks, extra, R)
+    if world > 1:
+        dist.destroy_process_group()
 
-    hbm_peak, peak_kind = read_peaks()
+
+def write_line(args, b, world, hbm_peak, peak_kind, stages, total_ms_max, units_all, n_steps, step_ms, emitted,
+               launches, lat_step, e2e_max, e2e_graph_ms, api_us, h2d, d2h, clocks, extra, R):
     a_bytes, s_bytes = attention_bytes(b), spec_bytes(b)
-    stages = {
-        "verify_attention": {"ms": ms_attn, "alg_bytes": a_bytes, "gbs": a_bytes / ms_attn / 1e6,
-                             "frac_of_measured_hbm": a_bytes / ms_attn / 1e6 / hbm_peak,
-                             "frac_of_8000": a_bytes / ms_attn / 1e6 / 8000.0},
-        "spec_verify": {"ms": ms_spec, "alg_bytes": s_bytes, "gbs": s_bytes / ms_spec / 1e6,
-                        "frac_of_measured_hbm": s_bytes / ms_spec / 1e6 / hbm_peak,
-                        "frac_of_8000": s_bytes / ms_spec / 1e6 / 8000.0},
-        "verify_attention_append": {"ms": ms_app, "note": "attention that also writes the verify tokens' K/V "
-                                                           "rows into their pages (same launch)"},
-        "spec_verify_sparse": {"ms": ms_sps, "alg_bytes": sparse_bytes(b),
-                               "gbs": sparse_bytes(b) / ms_sps / 1e6,
-                               "frac_of_measured_hbm": sparse_bytes(b) / ms_sps / 1e6 / hbm_peak,
-                               "note": "sparse draft payload, K = 64 table entries per draft row"},
-    }
+    stages["verify_attention"] = stage_entry(stages["verify_attention"], a_bytes, hbm_peak)
+    stages["spec_verify"] = stage_entry(stages["spec_verify"], s_bytes, hbm_peak)
+    stages["spec_verify_sparse"] = dict(stage_entry(stages["spec_verify_sparse"], sparse_bytes(b), hbm_peak),
+                                        note="sparse draft payload, K = 64 table entries per draft row")
+    stages["verify_attention_append"]["note"] = ("attention that also writes the verify tokens' K/V rows into "
+                                                 "their pages (same launch)")
     # The roofline is the single kernel with the longest launches: the attention
     # kernel (one launch per stage on this workload), ahead of each of the two
     # chained spec-verify kernels (see the ncu launch list under profiles/).
     dom = "verify_attention"
-    src = ["paper_2604_20919_gb300/csrc/attention_tc.cuh"]
     ds = stages[dom]
-    traffic = recorded_traffic(dom, source_hash(src))
-    cfg = workload_config(b, args.workload, args.seed)
-    cfg["l2"] = (f"inputs rotated over {R} device copies ({R * step_bytes / 1e6:.0f} MB > 2 x L2), "
-                 "K steps back to back as one CUDA graph replay")
-    cfg["parallelism"] = "replicas" if world > 1 else "single"
+    traffic = recorded_traffic(dom, source_hash(["paper_2604_20919_gb300/csrc/attention_tc.cuh"]))
+    ms_attn, ms_spec = stages["verify_attention"]["ms"], stages["spec_verify"]["ms"]
+    per_step = step_ms / n_steps
     line = {
         "metric": "verified tokens/s (one verification stage: attention + speculative sampling)",
         "value": units_all / (total_ms_max / 1000.0),
@@ -462,7 +591,11 @@ def run_dipsd(args):
         "ms_per_step": total_ms_max / n_steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "bf16", "data": "synthetic",
-        "config": cfg,
+        "config": bench_config(b, args.workload, args.seed, world),
+        "timing": {"replays": int(len(step_ms)), "steps_per_replay": n_steps,
+                   "ms_per_step_median": float(np.median(per_step)), "ms_per_step_min": float(per_step.min()),
+                   "ms_per_step_max": float(per_step.max()),
+                   "note": "value = median replay; every replay times exactly `steps` steps between CUDA events"},
         "emitted_tokens_per_step": emitted,
         "roofline": {"kernel": dom, "bound": "hbm", "achieved": ds["gbs"], "peak": hbm_peak, "unit": "GB/s",
                      "frac": ds["gbs"] / hbm_peak, "peak_kind": peak_kind, "traffic": traffic,
@@ -472,36 +605,32 @@ def run_dipsd(args):
             "value": emitted / ((64 * ms_attn + ms_spec) / 1000.0), "unit": "verified tokens/s",
             "note": "64 attention layers (each timed like verify_attention) + spec_verify; excludes every GEMM"},
         "step_latency_cold_l2_ms": lat_step,
-        "e2e": {"value": units_all / (e2e_max / 1000.0), "unit": "verified tokens/s",
-                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                "schedule": "per step: pinned H2D of q, logits, drafts; the call; D2H of "
-                            "accept_len, offsets, tokens; uploads overlap the previous step's compute",
-                "ms_per_step": e2e_max / args.steps},
+        "e2e": {"value": units_all / (e2e_max / 1000.0),
+                "unit": "verified tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "ms_per_step": e2e_max / n_steps, "api_host_us_per_call": api_us,
+                "schedule": "plain calls through the Python API (the library's validation and planning included); "
+                            "per step: pinned H2D of q, logits, drafts on a copy stream; the call; D2H of "
+                            "accept_len, offsets, tokens; uploads overlap the previous step's compute; host clock"},
+        "e2e_graph": {"value": emitted / (e2e_graph_ms / 1000.0), "unit": "verified tokens/s",
+                      "ms_per_step": e2e_graph_ms,
+                      "schedule": "the same steps captured as one CUDA graph of the API calls, replayed back to back"},
         "gpu_launches": int(launches),
         "clocks": clocks,
     }
+    line.update(extra)
     if world == 1 and args.cpu_seconds > 0:
         line["cpu_baseline"] = cpu_baseline(b, args.cpu_seconds)
     print(json.dumps(line), flush=True)
-    if world > 1:
-        dist.destroy_process_group()
 
 
-def run_pipeline(args):
+def measure_pipeline(args, dev):
     """Workload 5: 128 users in one KV pool dealt into 4 stages of 32, each stage
     one dipsd_verify_batch, stages alternating over two streams and rounds
-    repeating back to back (one CUDA graph); prints the sustained verified
-    tokens/s as its own line."""
+    repeating back to back (one CUDA graph); the sustained verified tokens/s."""
     import torch
     from paper_2604_20919_gb300 import dipsd
     from workloads import make_config, config_shape, CONFIG_NAMES
 
-    rank = int(os.environ.get("RANK", "0"))
-    if rank != 0:
-        return
-    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", "0")))
-    torch.cuda.set_device(dev)
-    dipsd.load()
     batches = make_config(5, seed=args.seed, device="cpu", kv_device=dev)
     s = config_shape(5, args.seed)
     L_all, ctx_all = s["L"], s["ctx"]
@@ -527,12 +656,11 @@ def run_pipeline(args):
                 with torch.cuda.stream(x["stream"]):
                     dipsd.dipsd_verify_batch(x["b"].members, L_all, ctx_all, x["q"], kc, vc, bt, x["b"].scale,
                                              x["z"], x["w"], x["d"], x["b"].seed, attn_out=x["attn"],
-                                             outputs=x["outs"],
-                                             ws=x["ws"], stream=x["stream"])
+                                             outputs=x["outs"], ws=x["ws"], stream=x["stream"])
         for sm in streams:
             cur.wait_stream(sm)
 
-    k = max(1, min(args.steps // 4, 200))
+    k = 20
     rounds(1)
     torch.cuda.synchronize()
     graph = torch.cuda.CUDAGraph()
@@ -540,28 +668,42 @@ def run_pipeline(args):
     with torch.cuda.graph(graph):
         rounds(k)
     launches = dipsd.dipsd_launch_count() - n0
-    for _ in range(max(1, args.warmup // 4)):
-        graph.replay()
-    torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(main)
     graph.replay()
-    e1.record(main)
     torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1)
+    first = replay_ms(graph, main, 1)[0]
+    reps = max(3, min(500, math.ceil(args.min_replay_ms / max(first, 1e-3))))
+    t = np.asarray(replay_ms(graph, main, reps)) / k
+    ms = float(np.median(t))
     emitted = sum(int(x["outs"][1][-1].item()) for x in stage)
     kv_bytes = sum(attention_bytes(x["b"]) for x in stage)
-    line = {
+    assert all(dipsd.device_status(x["ws"]) == 0 for x in stage)
+    res = {
         "metric": "verified tokens/s (sustained: 4 pipeline stages of 32 users on two streams)",
-        "value": emitted * k / (ms / 1000.0), "unit": "verified tokens/s", "n_gpus": 1,
-        "steps": k, "warmup": args.warmup, "ms_per_round": ms / k, "higher_is_better": True,
-        "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": CONFIG_NAMES[5], "stages": 4, "users_per_stage": 32, "streams": 2,
-                   "l2": "2 GB KV pool read once per round (>> L2)"},
-        "attention_gbs": kv_bytes * k / (ms / 1000.0) / 1e9,
-        "emitted_tokens_per_round": emitted, "gpu_launches": launches,
+        "value": emitted / (ms / 1000.0), "unit": "verified tokens/s", "ms_per_round": ms,
+        "ms_per_round_min": float(t.min()), "ms_per_round_max": float(t.max()), "replays": reps,
+        "rounds_per_replay": k, "config": {"workload": CONFIG_NAMES[5], "stages": 4, "users_per_stage": 32,
+                                           "streams": 2, "l2": "2 GB KV pool read once per round (>> L2)"},
+        "attention_gbs": kv_bytes / (ms / 1000.0) / 1e9,
+        "emitted_tokens_per_round": emitted, "gpu_launches_per_replay": launches,
     }
-    print(json.dumps(line), flush=True)
+    del stage, kc, vc, batches
+    torch.cuda.empty_cache()
+    return res
+
+
+def run_pipeline(args):
+    """`--workload 5`: the pipelined schedule's sustained rate as its own line."""
+    import torch
+    from paper_2604_20919_gb300 import dipsd
+    if int(os.environ.get("RANK", "0")) != 0:
+        return
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", "0")))
+    torch.cuda.set_device(dev)
+    dipsd.load()
+    res = measure_pipeline(args, dev)
+    res.update({"n_gpus": 1, "steps": res["rounds_per_replay"], "warmup": args.warmup, "higher_is_better": True,
+                "dtype": "bf16", "data": "synthetic"})
+    print(json.dumps(res), flush=True)
 
 
 def main():

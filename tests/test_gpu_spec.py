@@ -151,3 +151,16 @@ def test_spec_verify_output_law_monte_carlo(cuda_lib):
             alpha = np.minimum(p[k], q[k]).sum()
             sd = math.sqrt(alpha * (1 - alpha) / reached[k])
             assert abs(acc_hits[k] / reached[k] - alpha) < 4 * sd
+
+
+@pytest.mark.parametrize("nk1,nk2", [(4, 2), (8, 4), (16, 8)])
+def test_spec_verify_segment_sizes(cuda_lib, nk1, nk2):
+    """Every segment size of the two passes (16-byte vectors per lane): more or
+    fewer segments per row, ragged last segments, L = 0 and L = 31 users."""
+    rng = np.random.default_rng(30 + nk1)
+    L = np.concatenate([[0, 31], rng.integers(0, 9, size=40)])
+    b = make_batch(L, np.zeros_like(L), Hq=8, Hkv=1, D=64, V=20008, logit_std=1.5, noise_sigma=0.7,
+                   seed=30 + nk1, spec_only=True)
+    with cuda_lib.plan_override(spec_nk1=nk1, spec_nk2=nk2):
+        st = check_spec(b, *_run(cuda_lib, b))
+    print(f"segments {nk1}/{nk2}: {st}")
