@@ -121,14 +121,20 @@ int dipsd_verify_attention(int B, const int* h_L, const int* h_ctx,
                            void* d_out, void* d_workspace, size_t workspace_bytes,
                            void* stream);
 
-/* How a verify_attention launch cuts the batch into work items (host only:
- * no CUDA call, no device needed).  The attention entry points make the same
+/* How a verify_attention launch cuts the batch into work (host only: no
+ * CUDA call, no device needed).  The attention entry points make the same
  * plan for a device with num_sms SMs (append = 0: dipsd_verify_attention and
  * dipsd_verify_batch; append = 1: the *_append entry points).
  *
- * A work item is one (user, 128-row block of its G*(L_i+1) query rows, KV
- * head, KV split); a user's KV split s covers keys [s*split_len, (s+1)*split_len)
- * of its C_i+L_i+1, split_len a multiple of DIPSD_PAGE_SIZE.
+ * Either one CTA per work item: (user, 128-row block of its G*(L_i+1) query
+ * rows, KV head, KV split), a user's KV split s covering keys
+ * [s*split_len, (s+1)*split_len) of its C_i+L_i+1 (split_len a multiple of
+ * DIPSD_PAGE_SIZE); or (stream_chunks > 0) a persistent grid over page
+ * streams: the pages of every (user, row block, KV head) as one stream, the
+ * streams of users 0..B-1 (row block, then head, in order) back to back, cut
+ * into stream_chunks chunks (about equal pages plus a fixed charge per
+ * stream piece), CTA b taking chunk b; a stream cut by chunk boundaries has
+ * one split per chunk it touches, merged afterwards.
  *
  * B, h_L, h_ctx, Hq, Hkv, D   as for dipsd_verify_attention
  * num_sms       SMs of the device the plan is for (>= 1)
@@ -136,24 +142,27 @@ int dipsd_verify_attention(int B, const int* h_L, const int* h_ctx,
  * out           filled on success (caller-owned)
  * h_nsplit,
  * h_split_len   [B] host, nullable: per user the number of KV splits and the
- *               keys per split
+ *               keys per split (stream_chunks > 0: the most splits one of the
+ *               user's streams gets, and the keys of one of its streams)
+ * h_chunk_bound [num_sms + 1] host, nullable: stream_chunks > 0: chunk b is
+ *               pages [h_chunk_bound[b], h_chunk_bound[b + 1]) of the streams
  * Returns DIPSD_OK; the status dipsd_verify_attention would return for
  * invalid lengths or shapes; DIPSD_ERR_INVALID_ARG for num_sms < 1 or a null
  * out.  Nothing is written on failure.
  * ---------------------------------------------------------------------- */
 typedef struct {
-  int n_items;     /* work items */
-  int grid;        /* CTAs launched: n_items, or fewer (a persistent grid,
-                      CTA b walking items b, b + grid, b + 2 grid, ...) */
+  int n_items;     /* work items (page streams: the pieces of all chunks) */
+  int grid;        /* CTAs launched: n_items, or (chunk_pages > 0) the chunks */
   int cluster;     /* > 1: every user's KV in `cluster` splits that merge
                       inside one thread-block cluster; 0 otherwise */
-  int n_merge;     /* (verify token, query head) rows merged by the separate
-                      merge kernel after the grid (0: no merge launch) */
+  int n_merge;     /* (verify token, query head) rows the separate merge
+                      kernel visits after the grid (0: no merge launch) */
+  int stream_chunks; /* > 0: the persistent grid's chunks (CTAs) */
   size_t ws_bytes; /* workspace bytes of this plan past the status header */
 } dipsd_attention_plan;
 int dipsd_verify_attention_plan(int B, const int* h_L, const int* h_ctx, int Hq, int Hkv, int D,
                                 int num_sms, int append, dipsd_attention_plan* out,
-                                int* h_nsplit, int* h_split_len);
+                                int* h_nsplit, int* h_split_len, int* h_chunk_bound);
 
 /* ------------------------------------------------------------------------
  * Speculative verification (Sec. II-A stage 2: first-mismatch truncation and

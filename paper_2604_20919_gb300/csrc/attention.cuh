@@ -3,10 +3,23 @@
 // batch verification, Sec. II-A stage 2; the I*L term of Eq. (Fv)).
 //
 // This header holds what the attention kernel (attention_tc.cuh) shares with
-// the host: the work-item parameters (work item = user i, KV head h, row
-// block, KV split; rows r = t*G + g), and verify_attention_merge_kernel,
-// which combines the splits of one (user, head) through global memory when
+// the host: the work parameters (rows r = t*G + g of user i pack its verify
+// tokens and the G query heads of KV head h; a row block is 128 rows), the
+// decoding of a CTA's work, and verify_attention_merge_kernel, which combines
+// the KV splits of one (user, row block, head) through global memory when
 // they do not run as one cluster.
+//
+// Two ways to cut the work:
+//   * items (one per CTA): (user, row block, KV head, split), every split of
+//     a user `split_len` keys long;
+//   * page streams (a persistent grid of at most one CTA per SM): the keys of
+//     every (user, row block, KV head) as one stream of whole pages, the
+//     streams of all users back to back, cut into chunks [chunk_bound[b],
+//     chunk_bound[b + 1]), one per CTA.  A CTA takes the pieces of the
+//     streams its chunk covers, in order; the host cuts the chunks so that
+//     every CTA carries about the same pages plus a fixed cost per piece.  A
+//     stream cut by a chunk boundary is merged afterwards, its split s being
+//     its piece in the s-th chunk it touches.
 #pragma once
 
 #include "common.cuh"
@@ -14,6 +27,7 @@
 namespace dipsd {
 
 constexpr unsigned kDevErrBadBlock = 4u;  // an appended row's page id outside [0, num_blocks)
+constexpr int kMaxChunks = 256;           // CTAs of a grid over page streams
 
 struct AttnUser {
   int q_off;      // first verify token of the user in q / out
@@ -50,8 +64,11 @@ struct AttnParams {
                 // form one thread-block cluster and merge in shared memory
   int B, Hq, Hkv, G, max_blocks;
   int n_items, n_merge;
+  int n_chunks, total_pages;  // page streams (n_chunks > 0): chunks (CTAs), all pages
   float scale_log2;  // softmax_scale * log2(e)
   int item_off[CAP + 1];
+  int page_off[CAP + 1];  // page streams: first page of user i's streams
+  int chunk_bound[kMaxChunks + 1];  // page streams: chunk b is [chunk_bound[b], chunk_bound[b + 1])
   int merge_off[CAP + 1];
   long long part_off[CAP];  // first partial row of the user (multi-split users)
   AttnUser u[CAP];
@@ -67,9 +84,79 @@ __device__ __forceinline__ int find_user(const int* off, int B, int idx) {
   return lo;
 }
 
+// One unit of a CTA's work: keys [kv_begin, kv_end) of the stream of user
+// ui, row block rb and KV head h, which is split `split` of the stream's
+// `nsplit`; `next` is where the CTA's next unit starts (page streams).
+struct Work {
+  int ui, h, rb, split, nsplit, kv_begin, kv_end, next;
+};
+
+__device__ __forceinline__ int pages_of(const AttnUser& U) { return (U.kv_len + kPage - 1) / kPage; }
+
+// Item decoding: item = ((user, row block), head, split), split innermost.
+template <int CAP>
+__device__ __forceinline__ Work work_of_item(const AttnParams<CAP>& p, int item) {
+  Work w;
+  w.ui = find_user<CAP>(p.item_off, p.B, item);
+  const AttnUser& U = p.u[w.ui];
+  int local = item - p.item_off[w.ui];
+  w.split = local % U.nsplit;
+  local /= U.nsplit;
+  w.h = local % p.Hkv;
+  w.rb = local / p.Hkv;
+  w.nsplit = U.nsplit;
+  w.kv_begin = w.split * U.split_len;
+  w.kv_end = min(w.kv_begin + U.split_len, U.kv_len);
+  w.next = 0;
+  return w;
+}
+
+// The chunk that holds page `pos` (page streams).
+template <int CAP>
+__device__ __forceinline__ int chunk_of(const AttnParams<CAP>& p, int pos) {
+  int lo = 0, hi = p.n_chunks - 1;  // last b with chunk_bound[b] <= pos
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (p.chunk_bound[mid] <= pos) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+// Splits of the page stream that starts at page s0 and holds np pages: the
+// chunks it touches, the first of them c0.
+template <int CAP>
+__device__ __forceinline__ int stream_splits(const AttnParams<CAP>& p, int s0, int np, int* c0) {
+  *c0 = chunk_of<CAP>(p, s0);
+  return chunk_of<CAP>(p, s0 + np - 1) - *c0 + 1;
+}
+
+// Page-stream decoding: the piece that starts at page `pos` of CTA `cta`,
+// whose chunk ends at page `hi`.  Streams of user i: index (rb * Hkv + h),
+// each pages_of(U) pages.
+template <int CAP>
+__device__ __forceinline__ Work work_of_page(const AttnParams<CAP>& p, int pos, int cta, int hi) {
+  Work w;
+  w.ui = find_user<CAP>(p.page_off, p.B, pos);
+  const AttnUser& U = p.u[w.ui];
+  const int np = pages_of(U);
+  const int sidx = (pos - p.page_off[w.ui]) / np;
+  w.h = sidx % p.Hkv;
+  w.rb = sidx / p.Hkv;
+  const int s0 = p.page_off[w.ui] + sidx * np;
+  w.next = min(hi, s0 + np);
+  w.kv_begin = (pos - s0) * kPage;
+  w.kv_end = min((w.next - s0) * kPage, U.kv_len);
+  int c0;
+  w.nsplit = stream_splits<CAP>(p, s0, np, &c0);
+  w.split = cta - c0;
+  return w;
+}
+
 // Combines the KV splits of every (verify token, query head) row of users
 // with more than one split: m = max_s m_s, w_s = 2^(m_s - m),
-// out = sum_s w_s o_s / sum_s w_s l_s.  One warp per row.
+// out = sum_s w_s o_s / sum_s w_s l_s.  One warp per row: lane k holds the
+// (m, l) of splits k, k + 32, ..., the weights reach every lane by shuffle,
+// and the O rows of eight splits are loaded before any is used.
 template <int D, int CAP>
 __global__ void __launch_bounds__(128)
 verify_attention_merge_kernel(const __grid_constant__ AttnParams<CAP> p) {
@@ -84,31 +171,62 @@ verify_attention_merge_kernel(const __grid_constant__ AttnParams<CAP> p) {
   const int t = local / p.Hq, hq = local % p.Hq;
   const int h = hq / p.G, g = hq % p.G;
   const int M = p.G * U.T;
-  const int r = t * p.G + g;
-  float m = -INFINITY;
-  for (int s = 0; s < U.nsplit; ++s) {
-    const long long pr = p.part_off[ui] + static_cast<long long>(s * p.Hkv + h) * M + r;
-    m = fmaxf(m, p.part_ml[pr].x);
+  int ns = U.nsplit;
+  if (p.n_chunks > 0) {  // page streams: this row's stream may be whole
+    const int np = pages_of(U), sidx = ((t * p.G + g) / 128) * p.Hkv + h;
+    int c0;
+    ns = stream_splits<CAP>(p, p.page_off[ui] + sidx * np, np, &c0);
+    if (ns == 1) return;  // written by its CTA
   }
+  // partial row of split s: base + s * stride
+  const long long base = p.part_off[ui] + static_cast<long long>(h) * M + t * p.G + g;
+  const long long stride = static_cast<long long>(p.Hkv) * M;
+  float m = -INFINITY;
+  for (int s = lane; s < ns; s += 32) m = fmaxf(m, p.part_ml[base + s * stride].x);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
   constexpr int kPer = D / 32;
   float acc[kPer];
 #pragma unroll
   for (int k = 0; k < kPer; ++k) acc[k] = 0.f;
   float l = 0.f;
-  for (int s = 0; s < U.nsplit; ++s) {
-    const long long pr = p.part_off[ui] + static_cast<long long>(s * p.Hkv + h) * M + r;
-    const float2 ml = p.part_ml[pr];
-    const float w = ml.x == -INFINITY ? 0.f : fast_exp2(ml.x - m);
-    l += w * ml.y;
-    const float* po = p.part_o + pr * D + lane * kPer;
-    if constexpr (kPer == 4) {
-      const float4 v = *reinterpret_cast<const float4*>(po);
-      acc[0] += w * v.x; acc[1] += w * v.y; acc[2] += w * v.z; acc[3] += w * v.w;
-    } else {
-      const float2 v = *reinterpret_cast<const float2*>(po);
-      acc[0] += w * v.x; acc[1] += w * v.y;
+  for (int c0 = 0; c0 < ns; c0 += 32) {
+    // lane k: the weight of split c0 + k
+    float w = 0.f;
+    if (c0 + lane < ns) {
+      const float2 ml = p.part_ml[base + (c0 + lane) * stride];
+      w = ml.x == -INFINITY ? 0.f : fast_exp2(ml.x - m);
+      l += w * ml.y;
+    }
+    const int nc = min(32, ns - c0);
+    for (int k0 = 0; k0 < nc; k0 += 8) {
+      float v[8][kPer];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const float* po = p.part_o + (base + (c0 + k0 + k) * stride) * D + lane * kPer;
+        if (k0 + k < nc) {
+          if constexpr (kPer == 4) {
+            const float4 x = *reinterpret_cast<const float4*>(po);
+            v[k][0] = x.x; v[k][1] = x.y; v[k][2] = x.z; v[k][3] = x.w;
+          } else {
+            const float2 x = *reinterpret_cast<const float2*>(po);
+            v[k][0] = x.x; v[k][1] = x.y;
+          }
+        } else {
+#pragma unroll
+          for (int e = 0; e < kPer; ++e) v[k][e] = 0.f;
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const float wk = __shfl_sync(0xffffffffu, w, (k0 + k) & 31);
+#pragma unroll
+        for (int e = 0; e < kPer; ++e) acc[e] += wk * v[k][e];
+      }
     }
   }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) l += __shfl_xor_sync(0xffffffffu, l, o);
   const float inv = 1.f / l;
   __nv_bfloat16* out = p.out + (static_cast<size_t>(U.q_off + t) * p.Hq + hq) * D + lane * kPer;
 #pragma unroll

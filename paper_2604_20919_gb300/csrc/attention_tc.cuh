@@ -1,13 +1,15 @@
 // verify_attention on the 5th-generation tensor cores (tcgen05 + TMEM).
 //
-// Work decomposition: a work item is (user i, KV head h, row block, KV
-// split); rows r = t*G + g pack the G query heads of the KV group and the T_i
-// verify tokens (Sec. II-A stage 2: all L_i+1 tokens of a user are verified
-// in one pass), so each K/V byte brought on chip serves every row.  One CTA
-// per item, or (PERSIST) a grid of at most one CTA per SM in which CTA b
-// takes items b, b + gridDim.x, ...: the rings, the S/P buffers and every
-// barrier phase then run on across items, so the producer streams the next
-// item's tiles while the softmax warps finish the current one.
+// Work decomposition: rows r = t*G + g pack the G query heads of a KV group
+// and the T_i verify tokens of user i (Sec. II-A stage 2: all L_i+1 tokens of
+// a user are verified in one pass), so each K/V byte brought on chip serves
+// every row.  One CTA per work item (user, row block, KV head, KV split), or
+// (PERSIST) a grid of at most one CTA per SM over the page streams of every
+// (user, row block, KV head) laid back to back and cut into equal chunks of
+// pages (attention.cuh): CTA b takes the pieces of the streams its chunk
+// covers.  The rings, the S/P buffers and every barrier phase then run on
+// across pieces, so the producer streams the next piece's tiles while the
+// softmax warps finish the current one; every CTA carries the same pages.
 //
 // Roles (6 warps):
 //   warp 0      TMA producer into a ring of kStages 128-token K tiles and
@@ -51,7 +53,8 @@
 // of O, receives the other ranks' (m, l) rows and their rows of its chunks in
 // its drained K ring, and writes those columns of the output.
 // TMEM columns: S/P double buffer [0,128) [128,256), O [256, 256+D), Q
-// [384, 384 + D/2).  Shared memory holds only the two rings (Q and P live in
+// double buffer [384, 384 + D/2) [448, 448 + D/2) (item n's Q in buffer
+// n & 1, written one item ahead).  Shared memory holds only the two rings (Q and P live in
 // tensor memory, so no product re-reads an operand from shared memory every
 // tile), which leaves room for kStages tiles of K and of V in flight.
 #pragma once
@@ -65,6 +68,7 @@ constexpr int kTcThreads = 192;
 constexpr int kTcTile = 128;               // keys per tile (8 pages)
 constexpr uint32_t kTmemCols = 512;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
+constexpr uint32_t kQCols = 64;            // TMEM columns of one Q buffer (D / 2 bf16 pairs at most)
 
 template <int D>
 struct TcSmem {
@@ -92,8 +96,8 @@ static_assert(TcSmem<128>::kAlloc <= 232448 && TcSmem<64>::kAlloc <= 232448, "sh
 // tm_k: 4-D {64 columns, 16 rows, heads, blocks}, one 64-column half of a
 // page per box; tm_v: 5-D {64 columns, 16 rows, halves, heads, blocks}, a
 // whole page per box.
-// PERSIST: the grid is smaller than the item count and each CTA walks
-// several items; otherwise every CTA runs exactly one (the single-pass code).
+// PERSIST: every CTA walks the pieces of its chunk of the page streams;
+// otherwise every CTA runs exactly one item (the single-pass code).
 template <int D, int CAP, bool PERSIST>
 __global__ void __launch_bounds__(kTcThreads, 1)
 verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __grid_constant__ CUtensorMap tm_k,
@@ -114,36 +118,44 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
   uint64_t* p_full = s_full + 2;       // [2]
   uint64_t* pv_done = p_full + 2;      // [2]
   uint64_t* o_final = pv_done + 2;
-  uint64_t* q_ready = o_final + 1;
-  uint64_t* k_patch = q_ready + 1;   // [S] (each used at most once: new rows span <= 2 tiles)
+  uint64_t* q_ready = o_final + 1;   // [2]: one per Q buffer
+  uint64_t* k_patch = q_ready + 2;   // [S] (each used at most once: new rows span <= 2 tiles)
   uint64_t* v_patch = k_patch + S;   // [S]
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(v_patch + S);
 
-  // ---- work items: this CTA takes blockIdx.x, blockIdx.x + gridDim.x, ...
-  // (one item when the grid has an item per CTA).  Every role walks the same
-  // items in the same order; ring slots and barrier phases run on across
-  // items (global tile index g0 + j).
-  int ui, split, h, rb, M, row0, kv_begin, kv_end, ntiles, split_pages_n;
+  // ---- work: item blockIdx.x (one per CTA), or (PERSIST) the pieces of the
+  // page streams in this CTA's chunk [chunk_lo, chunk_hi), in order.  Every
+  // role walks the same pieces in the same order; ring slots and barrier
+  // phases run on across them (global tile index g0 + j).
+  const int chunk_lo = PERSIST ? p.chunk_bound[blockIdx.x] : static_cast<int>(blockIdx.x);
+  const int chunk_hi = PERSIST ? p.chunk_bound[blockIdx.x + 1] : 0;
+  auto decode = [&](int w) {
+    return PERSIST ? work_of_page<CAP>(p, w, blockIdx.x, chunk_hi) : work_of_item<CAP>(p, w);
+  };
+  int ui, split, nsplit, h, rb, M, row0, kv_begin, kv_end, ntiles, split_pages_n, next_w;
   AttnUser U;
-  auto set_item = [&](int item) {
-    ui = find_user<CAP>(p.item_off, p.B, item);
+  auto set_item = [&](int w) {
+    const Work W = decode(w);
+    ui = W.ui;
     U = p.u[ui];
-    int local = item - p.item_off[ui];
-    split = local % U.nsplit;
-    local /= U.nsplit;
-    h = local % p.Hkv;
-    rb = local / p.Hkv;
+    split = W.split;
+    nsplit = W.nsplit;
+    h = W.h;
+    rb = W.rb;
     M = p.G * U.T;
     row0 = rb * 128;
-    kv_begin = split * U.split_len;
-    kv_end = min(kv_begin + U.split_len, U.kv_len);
+    kv_begin = W.kv_begin;
+    kv_end = W.kv_end;
+    next_w = W.next;
     ntiles = max(0, (kv_end - kv_begin + kTcTile - 1) / kTcTile);  // 0: an empty split
     // Splits start on a page.  A split's last tile holds only the pages up
     // to kv_end: only those are loaded, multiplied (Q K^T with N = 16 per
     // page, one P V step per page) and run through the softmax.
     split_pages_n = (kv_end + kPage - 1) / kPage - kv_begin / kPage;
   };
-  set_item(blockIdx.x);
+  // is there work after the current unit (the loop tests it before set_item)
+  auto more = [&]() { return PERSIST && next_w < chunk_hi; };
+  set_item(chunk_lo);
   auto tile_pages = [&](int j) { return min(kTcTile / kPage, split_pages_n - j * (kTcTile / kPage)); };
   // tile j holds new (appended) rows: keys [max(key0, C_i), min(key0 + 128, kv_end)).
   // The patch barriers are single-use: a launch that appends runs one item per CTA.
@@ -167,7 +179,8 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
       mbar_init(&pv_done[b], 1);
     }
     mbar_init(o_final, 1);
-    mbar_init(q_ready, 4);
+    mbar_init(&q_ready[0], 4);
+    mbar_init(&q_ready[1], 4);
     for (int s = 0; s < S; ++s) {
       mbar_init(&k_patch[s], 1);
       mbar_init(&v_patch[s], 1);
@@ -186,6 +199,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  // Q of item n in buffer n & 1 (kQCols columns each)
   const uint32_t tS0 = tmem, tO = tmem + 2 * kTcTile, tQ = tmem + 384;
   float fin_m = -INFINITY, fin_l = 0.f;  // softmax threads: row state after the last tile
   bool fin_ok = false;
@@ -206,18 +220,27 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
     const int my_hf = kb % kHalves;
     int issued = 0;  // tiles issued over all items (the global tile index of the next)
     bool alive = true;
-    for (int item = blockIdx.x, n = 0; (PERSIST || n == 0) && item < p.n_items && alive; item += gridDim.x, ++n) {
-      if (n > 0) set_item(item);
+    // block ids of page group `group` of the split [kv_begin, kv_end) of the
+    // user whose block-table row is `row` (lane = page in the group)
+    auto fetch_of = [&](int row, int kb, int ke, int group) {
+      const int page = kb / kPage + group * 32 + lane;
+      return page < (ke + kPage - 1) / kPage ? __ldg(p.block_table + static_cast<size_t>(row) * p.max_blocks + page)
+                                             : p.num_blocks;  // past the split's end: never requested
+    };
+    int ahead = 0;  // the next unit's first page group, loaded one unit early
+    for (int n = 0; alive && (n == 0 || more()); ++n) {
+      if (n > 0) set_item(next_w);
       const int g0 = issued;
       const int* bt = p.block_table + static_cast<size_t>(U.bt_row) * p.max_blocks;
-      const int n_pages = (kv_end + kPage - 1) / kPage;  // pages of this split end here
-      const int page_base = kv_begin / kPage;
-      auto fetch = [&](int group) {
-        const int page = page_base + group * 32 + lane;
-        return page < n_pages ? __ldg(bt + page) : p.num_blocks;  // past the end: never requested
-      };
-      int cur = fetch(0);
+      auto fetch = [&](int group) { return fetch_of(U.bt_row, kv_begin, kv_end, group); };
+      int cur = n == 0 ? fetch(0) : ahead;
       int nxt = fetch(1);
+      if (more()) {
+        // the next unit's first page group, so its first loads do not wait
+        // on a dependent block-table read at the boundary
+        const Work Wn = decode(next_w);
+        ahead = fetch_of(p.u[Wn.ui].bt_row, Wn.kv_begin, Wn.kv_end, 0);
+      }
       for (int j = 0; j < ntiles; ++j) {
         const int gj = g0 + j;
         const int st = gj % S;
@@ -293,7 +316,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
       }
       // state update: the last split of the first row block writes the user's
       // new rows of head h into the pages
-      if (alive && p.new_k != nullptr && rb == 0 && split == U.nsplit - 1) {
+      if (alive && p.new_k != nullptr && rb == 0 && split == nsplit - 1) {
         const int n16 = U.T * (D / 8);
         for (int e = lane; e < n16; e += 32) {
           const int tt = e / (D / 8), c = e % (D / 8);
@@ -325,10 +348,11 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
       const uint32_t v_addr = smem_addr(sV);
       bool ok = true;
       int g0 = 0;  // global index of the item's first tile
-      for (int item = blockIdx.x, n = 0; (PERSIST || n == 0) && item < p.n_items && ok; item += gridDim.x, ++n) {
-        if (n > 0) set_item(item);
-        // Q of this item is in TMEM (written once the previous item's products were done)
-        ok = mbar_wait(q_ready, n & 1, p.status);
+      for (int n = 0; ok && (n == 0 || more()); ++n) {
+        if (n > 0) set_item(next_w);
+        // Q of this unit is in TMEM buffer n & 1 (written one unit ahead)
+        ok = mbar_wait(&q_ready[n & 1], (n >> 1) & 1, p.status);
+        const uint32_t tQn = tQ + (n & 1) * kQCols;
         int jq = 0, jp = 0;  // next Q K^T, next P V (within the item)
         uint64_t idle_since = 0;
         uint32_t idle_polls = 0;
@@ -346,7 +370,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
               const uint64_t bd = smem_desc_sw128(kt + (kk >> 2) * (kTcTile * 128) + (kk & 3) * 32, 0, 1024);
-              tc_mma_ts(tS0 + (gq & 1) * kTcTile, tQ + kk * 8, bd, id_qk, kk > 0 ? 1u : 0u);
+              tc_mma_ts(tS0 + (gq & 1) * kTcTile, tQn + kk * 8, bd, id_qk, kk > 0 ? 1u : 0u);
             }
             tc_commit(&s_full[gq & 1]);
             tc_commit(&k_empty[gq % S]);
@@ -399,37 +423,50 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
     const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;
     bool ok = true;
     int g0 = 0;  // global index of the item's first tile
-    for (int item = blockIdx.x, n = 0; (PERSIST || n == 0) && item < p.n_items && ok; item += gridDim.x, ++n) {
-      if (n > 0) set_item(item);
+    // Q row of the unit starting at w -> TMEM buffer qb, lane r, as bf16
+    // pairs (column c holds elements 2c, 2c+1); padding rows are zero
+    auto write_q = [&](int w, int qb) {
+      const Work Wj = decode(w);
+      const AttnUser Uj = p.u[Wj.ui];
+      const int hj = Wj.h, rgj = Wj.rb * 128 + r;
+      const bool validj = rgj < p.G * Uj.T;
+      tc_fence_after();
+      const uint4* qrow = reinterpret_cast<const uint4*>(
+          p.q + (static_cast<size_t>(Uj.q_off + rgj / p.G) * p.Hq + hj * p.G + rgj % p.G) * D);
+#pragma unroll
+      for (int cc = 0; cc < D / 64; ++cc) {
+        uint32_t w[32];
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          uint4 v = make_uint4(0, 0, 0, 0);
+          if (validj) v = __ldg(qrow + cc * 8 + c);
+          w[4 * c] = v.x;
+          w[4 * c + 1] = v.y;
+          w[4 * c + 2] = v.z;
+          w[4 * c + 3] = v.w;
+        }
+        tmem_st32(tQ + qb * kQCols + cc * 32 + lane_base, w);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&q_ready[qb]);
+    };
+    for (int n = 0; ok && (n == 0 || more()); ++n) {
+      if (n > 0) set_item(next_w);
       const int rg = row0 + r;  // row within the user
       const bool valid = rg < M;
       const int t = rg / p.G, g = rg % p.G;
 
-      // Q row -> TMEM lane r as bf16 pairs (column c holds elements 2c, 2c+1);
-      // padding rows are zero.  The previous item's products are done (its
-      // o_final was waited for), so its Q is no longer read.
-      {
-        tc_fence_after();
-        const uint4* qrow =
-            reinterpret_cast<const uint4*>(p.q + (static_cast<size_t>(U.q_off + t) * p.Hq + h * p.G + g) * D);
-#pragma unroll
-        for (int cc = 0; cc < D / 64; ++cc) {
-          uint32_t w[32];
-#pragma unroll
-          for (int c = 0; c < 8; ++c) {
-            uint4 v = make_uint4(0, 0, 0, 0);
-            if (valid) v = __ldg(qrow + cc * 8 + c);
-            w[4 * c] = v.x;
-            w[4 * c + 1] = v.y;
-            w[4 * c + 2] = v.z;
-            w[4 * c + 3] = v.w;
-          }
-          tmem_st32(tQ + cc * 32 + lane_base, w);
-        }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(q_ready);
-      }
+      // Q is written one item ahead, so the next item's Q K^T products can
+      // run while this item's last tiles and epilogue finish: item n + 1's Q
+      // goes to buffer (n + 1) & 1 once this item's first tile is softmaxed
+      // (off the path from this item's start to its first P V); the buffer's
+      // previous user, item n - 1, has its products done: its o_final was
+      // waited for.
+      if (n == 0) write_q(chunk_lo, 0);
+      const bool prefetch = more();
+      const int w_next = next_w;
+      if (prefetch && ntiles == 0) write_q(w_next, (n + 1) & 1);
 
       const int last_vis = min(U.ctx + t, kv_end - 1);  // last key of this row in this split
       // warps whose 32 rows are all padding write zero P, so every lane of P
@@ -534,6 +571,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&p_full[b]);
+        if (prefetch && j == 0) write_q(w_next, (n + 1) & 1);
       }
 
       // ---- epilogue: O row from TMEM
@@ -551,7 +589,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
           uint32_t o[32];
           tmem_ld32(tO + cc * 32 + lane_base, o);
           if (!valid) continue;
-          if (U.nsplit == 1) {
+          if (nsplit == 1) {
             uint4* dst = reinterpret_cast<uint4*>(orow + cc * 32);
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
@@ -567,7 +605,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
                                    __uint_as_float(o[4 * k + 2]), __uint_as_float(o[4 * k + 3]));
           }
         }
-        if (valid && U.nsplit > 1) p.part_ml[prow_idx] = make_float2(m, l);
+        if (valid && nsplit > 1) p.part_ml[prow_idx] = make_float2(m, l);
       }
       tc_fence_before();
       g0 += ntiles;

@@ -147,11 +147,13 @@ bool allow_smem(K kernel, int bytes, bool* done) {
 struct AttnPlan {
   int B = 0, Hq = 0, Hkv = 0, G = 0, D = 0;
   int n_items = 0, n_merge = 0;
+  int n_chunks = 0, total_pages = 0;  // page streams (persistent grid): chunks, all pages
+  std::vector<int> chunk_bound;        // chunk b: pages [chunk_bound[b], chunk_bound[b + 1])
   int grid = 0;     // CTAs launched: n_items, or fewer that each walk several items
   int cluster = 0;  // > 1: splits merged inside a thread-block cluster of this size
   long long part_rows = 0;
   std::vector<AttnUser> u;
-  std::vector<int> item_off, merge_off;
+  std::vector<int> item_off, merge_off, page_off;
   std::vector<long long> part_off;
   size_t ws_bytes = 0;  // attention region only (excludes the status word)
 };
@@ -180,6 +182,55 @@ int check_attn_users(int B, const int* L, const int* ctx, int Hq, int Hkv, int D
 // Costs are in units of 64 tokens of one (user, head) stream.
 // Pages per split when `pages` pages are cut into `ns` near-equal splits.
 static int split_pages(int pages, int ns) { return (pages + ns - 1) / ns; }
+
+// Chunks of the page streams (stream k holds np[k] pages; the streams back to
+// back) for at most `grid` CTAs, cut so that every CTA carries about the same
+// cost: a page costs 1, each piece (a stream or the part of one a chunk
+// holds) kPiecePages more.  A stream that would start with less than a piece's
+// cost of room left goes whole to the next chunk.  Cut points come from the
+// smallest per-chunk cost that needs at most `grid` chunks (bisection).
+constexpr long long kPiecePages = 18;  // ~3.5 us per piece at ~0.2 us per page
+static std::vector<int> cut_chunks(const std::vector<int>& np, int grid) {
+  auto cut = [&](long long cap, std::vector<int>* out) {
+    long long acc = 0, pos = 0;
+    int n = 1;
+    if (out) out->assign(1, 0);
+    for (int pages : np) {
+      if (acc > 0 && acc + kPiecePages >= cap) {  // start this stream in a new chunk
+        ++n;
+        if (out) out->push_back(static_cast<int>(pos));
+        acc = 0;
+      }
+      acc += kPiecePages;
+      long long rem = pages;
+      for (;;) {
+        const long long room = std::max<long long>(1, cap - acc);
+        if (rem <= room) {
+          acc += rem;
+          pos += rem;
+          break;
+        }
+        pos += room;
+        rem -= room;
+        ++n;
+        if (out) out->push_back(static_cast<int>(pos));
+        acc = kPiecePages;  // the rest of the stream: a new piece in the next chunk
+      }
+    }
+    if (out) out->push_back(static_cast<int>(pos));
+    return n;
+  };
+  long long total = 0;
+  for (int pages : np) total += pages + kPiecePages;
+  long long lo = 1, hi = total + kPiecePages;  // cut(hi) gives one chunk
+  while (lo < hi) {
+    const long long mid = (lo + hi) / 2;
+    if (cut(mid, nullptr) <= grid) hi = mid; else lo = mid + 1;
+  }
+  std::vector<int> bounds;
+  cut(lo, &bounds);
+  return bounds;
+}
 
 void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int Hq, int Hkv, int D,
                     int sms, AttnPlan& pl, bool persist_ok = true) {
@@ -247,93 +298,54 @@ void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int
   }
   pl.cluster = (forced_cluster > 0 || best_b < best) && best_cl > 1 ? best_cl : 0;
 
-  // Persistent grid (more items than CTA slots): each CTA walks items
-  // blockIdx.x, + grid, ... and its K/V ring streams on across item
-  // boundaries, so an item costs its tiles plus ~0.5 (the softmax epilogue
-  // and the next Q) and a CTA ~2 once (prologue, last epilogue).  Cost: the
-  // most loaded CTA of that static assignment, items in launch order.  Not
-  // with the KV append (single-use patch barriers) nor the cluster merge.
+  // Persistent grid over page streams: the pages of every (user, row block,
+  // KV head) as one stream, the streams back to back, cut into equal chunks
+  // of pages, one chunk per CTA (one CTA per SM).  Taken whenever one CTA per
+  // item would need more than one wave of CTAs (each wave pays its own ramp
+  // and drain, and the cost model above undercounts them: measured on the
+  // ragged 32-user batch, 87 us over six waves against 76 us for the same
+  // work as a persistent grid), or when a test forces it.  Not with the KV
+  // append (single-use patch barriers) nor the cluster merge.
   int persist_mode = -1;  // -1: by cost, 0: never, 1: whenever allowed
   int grid_cap = slots;
   if (const int v = plan_override(DIPSD_TEST_ATTN_PERSIST)) persist_mode = v == 1 ? 1 : 0;
   if (const int v = plan_override(DIPSD_TEST_ATTN_GRID)) grid_cap = std::max(1, std::min(slots, v));
-  int best_pc = 0;
-  double best_p = 1e300;
-  if (persist_ok && pl.cluster <= 1 && persist_mode != 0) {
-    // Per candidate: the split of every user, the item count and a lower
-    // bound on the most loaded CTA (the mean load); the exact static
-    // assignment is then costed in ascending bound order until the bound
-    // passes the best cost found (same choice as costing every candidate).
-    struct Cand {
-      int c, grid;
-      bool any_split;
-      double bound;
-    };
-    std::vector<Cand> cs;
-    for (int c : cands) {
-      if (forced > 0) c = forced;
-      long long items = 0;
-      double total = 0;
-      bool any_split = false;
-      for (int i = 0; i < B; ++i) {
-        const int tiles = (ctx[i] + L[i] + 1 + kTcTile - 1) / kTcTile;
-        const int pages = (ctx[i] + L[i] + 1 + kPage - 1) / kPage;
-        const int cc = std::max(1, std::min(c, tiles));
-        const int sp = split_pages(pages, (tiles + cc - 1) / cc);
-        const int ns = (pages + sp - 1) / sp;
-        const long long reps = static_cast<long long>((pl.G * (L[i] + 1) + rows_cta - 1) / rows_cta) * Hkv;
-        items += ns * reps;
-        total += reps * (pages * kPage / 64.0 + 0.5 * ns);
-        any_split = any_split || ns > 1;
-      }
-      if ((items > grid_cap || persist_mode > 0) && items <= 64ll * slots) {
-        const int grid = static_cast<int>(std::min<long long>(items, grid_cap));
-        cs.push_back({c, grid, any_split, 2.0 + total / grid + (any_split ? 3.0 : 0.0)});
-      }
-      if (forced > 0) break;
-    }
-    std::stable_sort(cs.begin(), cs.end(), [](const Cand& x, const Cand& y) { return x.bound < y.bound; });
-    std::vector<double> load;
-    int best_rank = 1 << 30;  // position in `cands` of the best candidate (ties: the first, as listed)
-    auto rank_of = [&](int c) {
-      return static_cast<int>(std::find(std::begin(cands), std::end(cands), c) - std::begin(cands));
-    };
-    for (const Cand& k : cs) {
-      if (k.bound > best_p + 1e-9) break;
-      load.assign(k.grid, 2.0);
-      int slot = 0;  // CTA of the next item: items go round-robin over the grid
-      for (int i = 0; i < B; ++i) {
-        const int tiles = (ctx[i] + L[i] + 1 + kTcTile - 1) / kTcTile;
-        const int pages = (ctx[i] + L[i] + 1 + kPage - 1) / kPage;
-        const int cc = std::max(1, std::min(k.c, tiles));
-        const int sp = split_pages(pages, (tiles + cc - 1) / cc);
-        const int ns = (pages + sp - 1) / sp;
-        const int reps = ((pl.G * (L[i] + 1) + rows_cta - 1) / rows_cta) * Hkv;  // (row block, head) pairs
-        const double full = sp * kPage / 64.0 + 0.5;                           // every split but the last
-        const double last = (pages - (ns - 1) * sp) * kPage / 64.0 + 0.5;
-        for (int r = 0; r < reps; ++r)
-          for (int sidx = 0; sidx < ns; ++sidx) {
-            load[slot] += sidx + 1 < ns ? full : last;
-            if (++slot == k.grid) slot = 0;
-          }
-      }
-      const double cost = *std::max_element(load.begin(), load.end()) + (k.any_split ? 3.0 : 0.0);
-      const int rank = rank_of(k.c);
-      if (cost < best_p - 1e-9 || (cost <= best_p + 1e-9 && rank < best_rank)) {
-        best_p = cost;
-        best_pc = k.c;
-        best_rank = rank;
-      }
-    }
+  long long total_pages = 0;
+  for (int i = 0; i < B; ++i) {
+    const int rb = (pl.G * (L[i] + 1) + rows_cta - 1) / rows_cta;
+    total_pages += static_cast<long long>(rb) * Hkv * ((ctx[i] + L[i] + 1 + kPage - 1) / kPage);
   }
-  const bool persist = best_pc > 0 && (persist_mode > 0 || best_p < best);
-  if (persist) best_c = best_pc;
+  // items of the best one-item-per-CTA plan
+  long long best_items = 0;
+  for (int i = 0; i < B; ++i) {
+    const int tiles = (ctx[i] + L[i] + 1 + kTcTile - 1) / kTcTile;
+    const int pages = (ctx[i] + L[i] + 1 + kPage - 1) / kPage;
+    const int cc = std::max(1, std::min(best_c, tiles));
+    const int sp = split_pages(pages, (tiles + cc - 1) / cc);
+    best_items += static_cast<long long>((pages + sp - 1) / sp) * ((pl.G * (L[i] + 1) + rows_cta - 1) / rows_cta) * Hkv;
+  }
+  int sk_grid = 0;
+  std::vector<int> sk_bound;
+  if (persist_ok && pl.cluster <= 1 && persist_mode != 0 && total_pages < (1ll << 30)) {
+    std::vector<int> np;
+    for (int i = 0; i < B; ++i) {
+      const int streams = ((pl.G * (L[i] + 1) + rows_cta - 1) / rows_cta) * Hkv;
+      np.insert(np.end(), streams, (ctx[i] + L[i] + 1 + kPage - 1) / kPage);
+    }
+    sk_bound = cut_chunks(np, static_cast<int>(std::min<long long>(std::min(grid_cap, kMaxChunks), total_pages)));
+    sk_grid = static_cast<int>(sk_bound.size()) - 1;
+  }
+  const bool persist = sk_grid > 0 && (persist_mode > 0 || best_items > slots);
 
   pl.u.assign(B, AttnUser{});
   pl.item_off.assign(B + 1, 0);
   pl.merge_off.assign(B + 1, 0);
+  pl.page_off.assign(B + 1, 0);
+  pl.n_chunks = persist ? sk_grid : 0;
+  pl.total_pages = persist ? static_cast<int>(total_pages) : 0;
+  if (persist) pl.chunk_bound = sk_bound;
   pl.part_off.assign(B, -1);
-  long long items = 0, merge = 0, part = 0;
+  long long items = 0, merge = 0, part = 0, pos_pages = 0;
   for (int i = 0; i < B; ++i) {
     AttnUser& U = pl.u[i];
     U.q_off = i == 0 ? 0 : pl.u[i - 1].q_off + pl.u[i - 1].T;
@@ -343,22 +355,38 @@ void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int
     U.bt_row = bt_rows ? bt_rows[i] : i;
     const int tiles = (U.kv_len + kTcTile - 1) / kTcTile;
     const int pages = (U.kv_len + kPage - 1) / kPage;
+    U.n_rb = (pl.G * U.T + rows_cta - 1) / rows_cta;
+    pl.item_off[i] = static_cast<int>(items);
+    pl.merge_off[i] = static_cast<int>(merge);
     int ns, sp;
-    if (pl.cluster > 1) {
+    if (persist) {
+      // page streams: the most chunks one of the user's streams touches, and
+      // (for the plan query) the user's pages; items = pieces
+      pl.page_off[i] = static_cast<int>(pos_pages);
+      auto chunk_at = [&](long long pos) {
+        return static_cast<int>(std::upper_bound(sk_bound.begin(), sk_bound.end() - 1, static_cast<int>(pos)) -
+                                sk_bound.begin()) - 1;
+      };
+      ns = 1;
+      for (int k = 0; k < U.n_rb * Hkv; ++k, pos_pages += pages) {
+        const int c = chunk_at(pos_pages + pages - 1) - chunk_at(pos_pages) + 1;
+        ns = std::max(ns, c);
+        items += c;
+      }
+      sp = pages;
+    } else if (pl.cluster > 1) {
       ns = pl.cluster;  // trailing splits may be empty when pages < C
       sp = split_pages(pages, ns);
+      items += static_cast<long long>(ns) * U.n_rb * Hkv;
     } else {
       const int cc = std::max(1, std::min(best_c, tiles));
       ns = (tiles + cc - 1) / cc;
       sp = split_pages(pages, ns);
       ns = (pages + sp - 1) / sp;
+      items += static_cast<long long>(ns) * U.n_rb * Hkv;
     }
     U.nsplit = ns;
     U.split_len = sp * kPage;
-    U.n_rb = (pl.G * U.T + rows_cta - 1) / rows_cta;
-    pl.item_off[i] = static_cast<int>(items);
-    pl.merge_off[i] = static_cast<int>(merge);
-    items += static_cast<long long>(ns) * U.n_rb * Hkv;
     if (ns > 1 && pl.cluster <= 1) {
       pl.part_off[i] = part;
       part += static_cast<long long>(ns) * Hkv * pl.G * U.T;
@@ -367,8 +395,9 @@ void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int
   }
   pl.item_off[B] = static_cast<int>(items);
   pl.merge_off[B] = static_cast<int>(merge);
+  pl.page_off[B] = static_cast<int>(pos_pages);
   pl.n_items = static_cast<int>(items);
-  pl.grid = persist ? std::min(pl.n_items, grid_cap) : pl.n_items;
+  pl.grid = persist ? sk_grid : pl.n_items;
   pl.n_merge = static_cast<int>(merge);
   pl.part_rows = part;
   pl.ws_bytes = part ? align_up(part * sizeof(float2), 256) + align_up(part * D * sizeof(float), 256) : 0;
@@ -393,15 +422,22 @@ void fill_attn_params(AttnParams<CAP>& p, const AttnPlan& pl, const void* q, voi
   p.cluster = pl.cluster;
   p.B = pl.B; p.Hq = pl.Hq; p.Hkv = pl.Hkv; p.G = pl.G; p.max_blocks = max_blocks;
   p.n_items = pl.n_items; p.n_merge = pl.n_merge;
+  p.n_chunks = pl.n_chunks; p.total_pages = pl.total_pages;
+  if (pl.n_chunks > 0)
+    for (int b = 0; b <= pl.n_chunks; ++b) p.chunk_bound[b] = pl.chunk_bound[b];
   p.scale_log2 = scale * 1.4426950408889634f;
-  for (int i = 0; i <= pl.B; ++i) { p.item_off[i] = pl.item_off[i]; p.merge_off[i] = pl.merge_off[i]; }
+  for (int i = 0; i <= pl.B; ++i) {
+    p.item_off[i] = pl.item_off[i];
+    p.merge_off[i] = pl.merge_off[i];
+    p.page_off[i] = pl.page_off[i];
+  }
   for (int i = 0; i < pl.B; ++i) { p.part_off[i] = pl.part_off[i]; p.u[i] = pl.u[i]; }
 }
 
 template <int D, int CAP>
 int launch_attention_tc_t(const AttnPlan& pl, const AttnParams<CAP>& p, const CUtensorMap& tk,
                           const CUtensorMap& tv, cudaStream_t s, bool pdl) {
-  const bool persist = pl.grid < pl.n_items;
+  const bool persist = pl.n_chunks > 0;
   auto kern = persist ? verify_attention_tc_kernel<D, CAP, true> : verify_attention_tc_kernel<D, CAP, false>;
   static std::mutex mu;
   static bool attr_done[2][64] = {};
@@ -846,7 +882,8 @@ static int verify_attention_impl(int B, const int* h_L, const int* h_ctx, const 
 }
 
 int dipsd_verify_attention_plan(int B, const int* h_L, const int* h_ctx, int Hq, int Hkv, int D, int num_sms,
-                                int append, dipsd_attention_plan* out, int* h_nsplit, int* h_split_len) {
+                                int append, dipsd_attention_plan* out, int* h_nsplit, int* h_split_len,
+                                int* h_chunk_bound) {
   const int st = check_attn_users(B, h_L, h_ctx, Hq, Hkv, D);
   if (st != DIPSD_OK) return st;
   if (num_sms < 1 || !out) return DIPSD_ERR_INVALID_ARG;
@@ -856,6 +893,9 @@ int dipsd_verify_attention_plan(int B, const int* h_L, const int* h_ctx, int Hq,
   out->grid = pl.grid;
   out->cluster = pl.cluster > 1 ? pl.cluster : 0;
   out->n_merge = pl.n_merge;
+  out->stream_chunks = pl.n_chunks;
+  if (h_chunk_bound && pl.n_chunks > 0)
+    for (int b = 0; b <= pl.n_chunks; ++b) h_chunk_bound[b] = pl.chunk_bound[b];
   out->ws_bytes = pl.ws_bytes;
   for (int i = 0; i < B; ++i) {
     if (h_nsplit) h_nsplit[i] = pl.u[i].nsplit;

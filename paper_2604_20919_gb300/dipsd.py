@@ -53,7 +53,8 @@ _u64 = ctypes.c_uint64
 
 class AttentionPlan(ctypes.Structure):
     """dipsd_attention_plan of include/dipsd.h."""
-    _fields_ = [("n_items", _i), ("grid", _i), ("cluster", _i), ("n_merge", _i), ("ws_bytes", _sz)]
+    _fields_ = [("n_items", _i), ("grid", _i), ("cluster", _i), ("n_merge", _i), ("stream_chunks", _i),
+                ("ws_bytes", _sz)]
 
 
 class DipsdError(RuntimeError):
@@ -104,7 +105,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
                                              _vp, _vp, _vp, _sz, _vp]
     lib.dipsd_verify_attention_plan.restype = _i
     lib.dipsd_verify_attention_plan.argtypes = [_i, _i32p, _i32p, _i, _i, _i, _i, _i,
-                                                ctypes.POINTER(AttentionPlan), _i32p, _i32p]
+                                                ctypes.POINTER(AttentionPlan), _i32p, _i32p, _i32p]
     lib.dipsd_spec_verify_noalloc.restype = _i
     lib.dipsd_spec_verify_noalloc.argtypes = [_i, _i32p, _i32p, _u64, _i, _i, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
                                               _vp]
@@ -195,18 +196,21 @@ def dipsd_verify_attention_workspace_size(L, ctx, Hq: int, Hkv: int, D: int) -> 
 
 
 def dipsd_verify_attention_plan(L, ctx, Hq: int, Hkv: int, D: int, num_sms: int, append: bool = False) -> dict:
-    """The work-item plan the attention entry points make for a device with
+    """The work plan the attention entry points make for a device with
     num_sms SMs (host only).  Returns n_items, grid, cluster, n_merge,
-    ws_bytes and per user nsplit and split_len."""
+    stream_chunks, ws_bytes, per user nsplit and split_len, and (page-stream
+    plans) chunk_bound."""
     a, pa = _host_i32(L)
     b, pb = _host_i32(ctx)
     plan = AttentionPlan()
     nsplit, pn = _host_i32(np.zeros(len(a)))
     split_len, ps = _host_i32(np.zeros(len(a)))
+    bounds, pbd = _host_i32(np.zeros(int(num_sms) + 1))
     _check(load().dipsd_verify_attention_plan(len(a), pa, pb, Hq, Hkv, D, int(num_sms), 1 if append else 0,
-                                              ctypes.byref(plan), pn, ps), "dipsd_verify_attention_plan")
+                                              ctypes.byref(plan), pn, ps, pbd), "dipsd_verify_attention_plan")
     return {"n_items": plan.n_items, "grid": plan.grid, "cluster": plan.cluster, "n_merge": plan.n_merge,
-            "ws_bytes": int(plan.ws_bytes), "nsplit": nsplit, "split_len": split_len}
+            "stream_chunks": plan.stream_chunks, "ws_bytes": int(plan.ws_bytes), "nsplit": nsplit,
+            "split_len": split_len, "chunk_bound": bounds[:plan.stream_chunks + 1] if plan.stream_chunks else None}
 
 
 def dipsd_verify_attention(L, ctx, q, k_cache, v_cache, block_table, softmax_scale: float, out=None,

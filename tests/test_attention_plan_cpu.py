@@ -21,6 +21,14 @@ def dipsd():
     return d
 
 
+def _page_streams(L, ctx, G, Hkv):
+    """(user, pages) of every (user, row block, KV head) stream, in the order
+    the persistent grid lays them back to back."""
+    pages = -(-(np.asarray(ctx) + np.asarray(L) + 1) // PAGE)
+    rb = -(-(G * (np.asarray(L) + 1)) // ROWS_PER_ITEM)
+    return [(i, int(pages[i])) for i in range(len(L)) for _ in range(int(rb[i]) * Hkv)]
+
+
 def _check_plan(p, L, ctx, Hq, Hkv, D, num_sms, append, forced_cluster=False):
     L, ctx = np.asarray(L), np.asarray(ctx)
     G = Hq // Hkv
@@ -28,28 +36,45 @@ def _check_plan(p, L, ctx, Hq, Hkv, D, num_sms, append, forced_cluster=False):
     ns, sl = p["nsplit"], p["split_len"]
     assert (sl % PAGE == 0).all() and (sl >= PAGE).all()
     assert (ns >= 1).all()
-    # every key of a user lies in exactly one split; only cluster plans may
-    # carry trailing empty splits (every user then has exactly `cluster`)
-    assert (ns * sl >= kv_len).all()
-    if p["cluster"]:
-        assert p["cluster"] <= (3 if D == 128 else 6)
-        assert (ns == p["cluster"]).all()
-        assert p["n_merge"] == 0
-        # chosen by cost only when every cluster is resident at once
-        assert forced_cluster or p["n_items"] <= num_sms
-    else:
-        assert ((ns - 1) * sl < kv_len).all()
-    row_blocks = -(-(G * (L + 1)) // ROWS_PER_ITEM)
-    assert p["n_items"] == int((ns * row_blocks * Hkv).sum())
-    # the grid: one CTA per item, or a persistent grid of at most one CTA per SM
-    assert 1 <= p["grid"] <= p["n_items"]
-    if p["grid"] < p["n_items"]:
+    if p["stream_chunks"]:
+        # persistent grid over page streams, modelled here independently: the
+        # streams back to back, chunk b = pages [bound[b], bound[b + 1]) for
+        # CTA b; a stream has one split per chunk it touches
         assert not append and not p["cluster"]
-        assert p["grid"] <= num_sms
-    # multi-split users without a cluster go through the merge kernel: one
-    # merged row per (verify token, query head), (m, l) and D partial outputs
-    # per (split, head, row) in the workspace
-    split_users = (ns > 1) if not p["cluster"] else np.zeros_like(ns, dtype=bool)
+        bound = np.asarray(p["chunk_bound"])
+        streams = _page_streams(L, ctx, G, Hkv)
+        total = sum(n for _, n in streams)
+        assert p["grid"] == p["stream_chunks"] == len(bound) - 1 <= min(num_sms, 256)
+        assert bound[0] == 0 and bound[-1] == total and (np.diff(bound) > 0).all()
+        chunk_of = lambda pos: int(np.searchsorted(bound, pos, side="right")) - 1
+        pieces, ns_user, pos = 0, np.ones(len(L), dtype=int), 0
+        for i, n in streams:
+            c = chunk_of(pos + n - 1) - chunk_of(pos) + 1
+            pieces += c
+            ns_user[i] = max(ns_user[i], c)
+            pos += n
+        assert p["n_items"] == pieces
+        np.testing.assert_array_equal(ns, ns_user)
+        split_users = ns_user > 1
+    else:
+        # every key of a user lies in exactly one split; only cluster plans may
+        # carry trailing empty splits (every user then has exactly `cluster`)
+        assert (ns * sl >= kv_len).all()
+        if p["cluster"]:
+            assert p["cluster"] <= (3 if D == 128 else 6)
+            assert (ns == p["cluster"]).all()
+            assert p["n_merge"] == 0
+            # chosen by cost only when every cluster is resident at once
+            assert forced_cluster or p["n_items"] <= num_sms
+        else:
+            assert ((ns - 1) * sl < kv_len).all()
+        row_blocks = -(-(G * (L + 1)) // ROWS_PER_ITEM)
+        assert p["n_items"] == int((ns * row_blocks * Hkv).sum())
+        assert p["grid"] == p["n_items"]  # one CTA per item
+        split_users = (ns > 1) if not p["cluster"] else np.zeros_like(ns, dtype=bool)
+    # split users without a cluster go through the merge kernel: it visits one
+    # row per (verify token, query head); (m, l) and D partial outputs per
+    # (split, head, row) in the workspace
     assert p["n_merge"] == int(((L + 1) * Hq)[split_users].sum())
     part_rows = int((ns * Hkv * G * (L + 1))[split_users].sum())
     assert p["ws_bytes"] >= part_rows * (8 + 4 * D)
@@ -75,14 +100,14 @@ def test_plan_invariants_on_random_batches(dipsd, seed, num_sms):
 def test_plan_of_the_workloads(dipsd):
     """Workload 2 (8 users x 1024 tokens): 2 splits per (user, head) merged in
     a 2-CTA cluster, 128 CTAs, no merge launch.  Workload 3 (32 ragged users):
-    more items than SMs, so a persistent grid of one CTA per SM; the append
+    a persistent grid of one CTA per SM over the page streams; the append
     variant keeps one CTA per item."""
     s = config_shape(2, 0)
     p = dipsd.dipsd_verify_attention_plan(s["L"], s["ctx"], s["Hq"], s["Hkv"], s["D"], 152)
     assert (p["cluster"], p["n_items"], p["grid"], p["n_merge"]) == (2, 128, 128, 0)
     s = config_shape(3, 0)
     p = dipsd.dipsd_verify_attention_plan(s["L"], s["ctx"], s["Hq"], s["Hkv"], s["D"], 152)
-    assert p["cluster"] == 0 and p["n_items"] > 152 and p["grid"] == 152
+    assert p["cluster"] == 0 and p["stream_chunks"] > 0 and 140 <= p["grid"] <= 152
     pa = dipsd.dipsd_verify_attention_plan(s["L"], s["ctx"], s["Hq"], s["Hkv"], s["D"], 152, append=True)
     assert pa["grid"] == pa["n_items"]
     for cfg in (1, 2, 3, 4):
