@@ -11,7 +11,7 @@ import pytest
 import torch
 
 import oracle
-from parity import check_attention, valid_spec_outputs
+from parity import attention_reference, check_attention, valid_spec_outputs
 from workloads import make_batch, make_config
 
 pytestmark = pytest.mark.gpu
@@ -36,8 +36,8 @@ def _split_new_rows(b):
 
 
 def _reference(b):
-    return oracle.verify_attention(b.q.double().numpy(), b.k_cache.double().numpy(), b.v_cache.double().numpy(),
-                                   b.block_table.numpy(), b.ctx, b.L, b.scale)
+    """(oracle output, oracle attention of |V|) on the untouched cache."""
+    return attention_reference(b)
 
 
 def _append_run(dipsd, b):
@@ -58,7 +58,7 @@ def _append_run(dipsd, b):
 @pytest.mark.parametrize("cfg", [1, 2])
 def test_append_attention_workloads(cuda_lib, cfg):
     b = make_config(cfg, seed=3)
-    check_attention(_append_run(cuda_lib, b), _reference(b))
+    check_attention(_append_run(cuda_lib, b), *_reference(b))
 
 
 @pytest.mark.parametrize("L,ctx,Hq,Hkv,D", [
@@ -68,7 +68,7 @@ def test_append_attention_workloads(cuda_lib, cfg):
 ])
 def test_append_attention_edges(cuda_lib, L, ctx, Hq, Hkv, D):
     b = make_batch(L, ctx, Hq=Hq, Hkv=Hkv, D=D, V=64, seed=40 + sum(L))
-    check_attention(_append_run(cuda_lib, b), _reference(b))
+    check_attention(_append_run(cuda_lib, b), *_reference(b))
 
 
 @pytest.mark.parametrize("override,val", [("attn_split_tiles", 1), ("attn_split_tiles", 3), ("attn_cluster", 3),
@@ -78,7 +78,7 @@ def test_append_with_splits(cuda_lib, override, val):
     b = make_batch([31, 5, 0, 12], [50, 1000, 63, 200], Hq=64, Hkv=8, D=128, V=64, seed=47)
     with cuda_lib.plan_override(**{override: val}):
         out = _append_run(cuda_lib, b)
-    check_attention(out, _reference(b))
+    check_attention(out, *_reference(b))
 
 
 def test_batch_append_matches_batch(cuda_lib):

@@ -4,7 +4,7 @@ import pytest
 import torch
 
 import oracle
-from parity import attention_subset_reference, check_attention
+from parity import attention_reference, attention_subset_reference, check_attention, peaked_attention
 from workloads import make_batch, make_config
 
 pytestmark = pytest.mark.gpu
@@ -20,14 +20,14 @@ def _run(dipsd, b, ws=None):
 
 
 def _full_reference(b):
-    return oracle.verify_attention(b.q.double().numpy(), b.k_cache.double().numpy(), b.v_cache.double().numpy(),
-                                   b.block_table.numpy(), b.ctx, b.L, b.scale)
+    """(oracle output, oracle attention of |V|) of the whole batch."""
+    return attention_reference(b)
 
 
 @pytest.mark.parametrize("cfg", [1, 2, 3])
 def test_attention_workloads(cuda_lib, cfg):
     b = make_config(cfg, seed=0)
-    err = check_attention(_run(cuda_lib, b), _full_reference(b))
+    err = check_attention(_run(cuda_lib, b), *_full_reference(b))
     print(f"workload {cfg}: max abs err {err:.3e}")
 
 
@@ -36,9 +36,30 @@ def test_attention_long_context_sampled_users(cuda_lib):
     b = make_config(4, seed=0, device="cpu", kv_device=DEV)
     out = _run(cuda_lib, b)
     for users in ([0, 37], [63]):
-        rows, ref = attention_subset_reference(b, users)
-        err = check_attention(out[torch.from_numpy(rows).to(DEV)], ref)
+        rows, ref, ref_abs = attention_subset_reference(b, users, with_abs=True)
+        err = check_attention(out[torch.from_numpy(rows).to(DEV)], ref, ref_abs)
         print(f"workload 4 users {users}: max abs err {err:.3e}")
+    del b, out
+    torch.cuda.empty_cache()
+
+
+def test_attention_peaked_headline_shapes(cuda_lib):
+    """Workload 2's shapes (ctx 1024, 64/8/128) with peaked attention (Q x4,
+    V of mean 1): a single key counted or missed moves outputs by O(0.1 .. 1),
+    far outside both bounds (the CPU test of the parity check shows a causal
+    off-by-one and a dropped last page failing on these shapes)."""
+    b = peaked_attention(make_config(2, seed=6))
+    err = check_attention(_run(cuda_lib, b), *_full_reference(b))
+    print(f"peaked workload 2: max abs err {err:.3e}")
+
+
+def test_attention_peaked_long_context_sampled_users(cuda_lib):
+    """Workload 4 (ctx 32768) with peaked attention; oracle on sampled users."""
+    b = peaked_attention(make_config(4, seed=0, device="cpu", kv_device=DEV))
+    out = _run(cuda_lib, b)
+    rows, ref, ref_abs = attention_subset_reference(b, [5, 50], with_abs=True)
+    err = check_attention(out[torch.from_numpy(rows).to(DEV)], ref, ref_abs)
+    print(f"peaked workload 4: max abs err {err:.3e}")
     del b, out
     torch.cuda.empty_cache()
 
@@ -55,7 +76,7 @@ def test_attention_long_context_sampled_users(cuda_lib):
 ])
 def test_attention_edge_shapes(cuda_lib, L, ctx, Hq, Hkv, D):
     b = make_batch(L, ctx, Hq=Hq, Hkv=Hkv, D=D, V=64, seed=sum(L) + sum(ctx))
-    check_attention(_run(cuda_lib, b), _full_reference(b))
+    check_attention(_run(cuda_lib, b), *_full_reference(b))
 
 
 @pytest.mark.parametrize("split_tiles", [1, 2, 7])
@@ -64,7 +85,7 @@ def test_attention_forced_splits(cuda_lib, split_tiles):
     b = make_batch([5, 0, 8, 2], [1500, 3000, 333, 64], Hq=64, Hkv=8, D=128, V=64, seed=21)
     with cuda_lib.plan_override(attn_split_tiles=split_tiles):
         out = _run(cuda_lib, b)
-    check_attention(out, _full_reference(b))
+    check_attention(out, *_full_reference(b))
 
 
 @pytest.mark.parametrize("cluster,D", [(2, 128), (3, 128), (6, 64)])
@@ -75,7 +96,7 @@ def test_attention_cluster_merge(cuda_lib, cluster, D):
                    D=D, V=64, seed=23)
     with cuda_lib.plan_override(attn_cluster=cluster):
         out = _run(cuda_lib, b)
-    check_attention(out, _full_reference(b))
+    check_attention(out, *_full_reference(b))
 
 
 @pytest.mark.parametrize("grid,split_tiles,D", [(1, 0, 128), (3, 0, 128), (7, 2, 128), (5, 1, 64), (152, 1, 128)])
@@ -90,7 +111,7 @@ def test_attention_persistent_grid(cuda_lib, grid, split_tiles, D):
         ws = cuda_lib.workspace(cuda_lib.dipsd_verify_attention_workspace_size(b.L, b.ctx, b.Hq, b.Hkv, b.D), DEV)
         out = _run(cuda_lib, b, ws)
         assert cuda_lib.device_status(ws) == 0
-    check_attention(out, _full_reference(b))
+    check_attention(out, *_full_reference(b))
 
 
 def test_attention_ignores_slots_past_kv_len(cuda_lib):
@@ -111,7 +132,7 @@ def test_attention_ignores_slots_past_kv_len(cuda_lib):
             kc[blk] = float("nan")
             vc[blk] = float("nan")
     b.k_cache, b.v_cache = kc, vc
-    check_attention(_run(cuda_lib, b), ref)
+    check_attention(_run(cuda_lib, b), *ref)
 
 
 def test_attention_status_word_stays_clear(cuda_lib):

@@ -35,8 +35,8 @@ def test_pipelined_stages_on_two_streams(cuda_lib):
     for n, (b, (attn, acc, offs, toks, probs)) in enumerate(zip(batches, results)):
         st = check_spec(b, acc, offs, toks, probs)
         users = [0, int(np.argmax(b.ctx)), b.B - 1]
-        rows, ref = attention_subset_reference(b, users)
-        err = check_attention(attn[torch.from_numpy(rows).to(DEV)], ref)
+        rows, ref, ref_abs = attention_subset_reference(b, users, with_abs=True)
+        err = check_attention(attn[torch.from_numpy(rows).to(DEV)], ref, ref_abs)
         print(f"stage {n}: {st}, attention max err {err:.3e}")
 
 
@@ -74,5 +74,7 @@ def test_batch_with_permuted_membership(cuda_lib):
     torch.cuda.synchronize()
     ref = oracle.verify_attention(b.q.double().numpy(), b.k_cache.double().numpy(), b.v_cache.double().numpy(),
                                   b.block_table.numpy(), b.ctx, b.L, b.scale)
-    check_attention(attn, ref)
+    ref_abs = oracle.verify_attention(b.q.double().numpy(), b.k_cache.double().numpy(),
+                                      np.abs(b.v_cache.double().numpy()), b.block_table.numpy(), b.ctx, b.L, b.scale)
+    check_attention(attn, ref, ref_abs)
     check_spec(b, acc, offs, toks, probs)
