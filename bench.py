@@ -259,6 +259,24 @@ def run_reference(args):
 
 
 # --------------------------------------------------------------- timing
+def packed_layout(tensors, align=256):
+    """One uint8 buffer holding the tensors back to back (each at a 256-byte
+    aligned offset), and a function that returns their views into any buffer
+    of that layout."""
+    import torch
+    offs, n = [], 0
+    for t in tensors:
+        offs.append(n)
+        n += -(-(t.numel() * t.element_size()) // align) * align
+    buf = torch.zeros(n, dtype=torch.uint8)
+    for t, o in zip(tensors, offs):
+        buf[o:o + t.numel() * t.element_size()].copy_(t.contiguous().view(-1).view(torch.uint8))
+
+    def views_of(x):
+        return [x[o:o + t.numel() * t.element_size()].view(t.dtype).view(t.shape) for t, o in zip(tensors, offs)]
+    return buf, views_of
+
+
 def capture(fn, n, R, stream):
     """A CUDA graph of n consecutive calls fn(0), .., fn(n - 1) (lazy set-up
     settled outside the capture) and the library kernels one replay launches."""
@@ -482,40 +500,44 @@ def run_dipsd(args):
     lat_step = cold_latency(step, min(args.steps, 50))
 
     # end to end through the Python API: every step copies its inputs from
-    # pinned host memory into one of the R device copies (copy stream), makes
-    # the call and reads its results back into per-copy pinned buffers
-    # (compute stream); step k+1's upload overlaps step k's compute.
-    pin = lambda t: t.cpu().pin_memory()
-    keys = ("q", "z", "w", "d")
-    h_in = [pin(x) for x in (b.q, b.target_logits, b.draft_logits, b.draft_tokens)]
-    h_out = [[torch.empty_like(x, device="cpu").pin_memory() for x in outs[:3]] for _ in range(R)]
-    h2d = sum(x.numel() * x.element_size() for x in h_in)
-    d2h = sum(x.numel() * x.element_size() for x in h_out[0])
+    # pinned host memory into one of R device slots (copy stream), makes the
+    # call and reads its results back into that slot's pinned buffer (compute
+    # stream); step k+1's upload overlaps step k's compute.  A slot's inputs
+    # (q, target and draft logits, drafted tokens) sit back to back in one
+    # device buffer, and the results (accept_len, out_offsets, out_tokens) in
+    # another, so each step is one host-to-device and one device-to-host copy.
+    h_in, views_of = packed_layout([b.q, b.target_logits, b.draft_logits, b.draft_tokens])
+    h_in = h_in.pin_memory()
+    d_in = [torch.empty_like(h_in, device=dev) for _ in range(R)]
+    e_in = [dict(zip(("q", "z", "w", "d"), views_of(x))) for x in d_in]
+    o_host, o_views = packed_layout([x.cpu() for x in outs[:3]])
+    d_out = torch.empty_like(o_host, device=dev)
+    e_outs = tuple(o_views(d_out)) + (outs[3],)
+    h_out = [torch.empty_like(o_host).pin_memory() for _ in range(R)]
+    h2d, d2h = h_in.numel(), d_out.numel()  # bytes copied per step (the packed buffers)
     cs = torch.cuda.Stream()
+    ev_up = [torch.cuda.Event() for _ in range(R)]
+    ev_free = [torch.cuda.Event() for _ in range(R)]
     api_s = [0.0]
 
     def e2e_steps(n, host_clock=False):
-        free = [None] * R
         cs.wait_stream(stream)
         for i in range(n):
             k = i % R
-            c = copies[k]
+            c = e_in[k]
+            if i >= R:
+                cs.wait_event(ev_free[k])
             with torch.cuda.stream(cs):
-                if free[k] is not None:
-                    cs.wait_event(free[k])
-                for hd, key in zip(h_in, keys):
-                    c[key].copy_(hd, non_blocking=True)
-                up = torch.cuda.Event()
-                up.record(cs)
-            stream.wait_event(up)
+                d_in[k].copy_(h_in, non_blocking=True)
+            ev_up[k].record(cs)
+            stream.wait_event(ev_up[k])
             t0 = time.perf_counter()
-            step(k)
+            dipsd.dipsd_verify_batch(b.members, b.L, b.ctx, c["q"], copies[k]["kc"], copies[k]["vc"], bt, b.scale,
+                                     c["z"], c["w"], c["d"], b.seed, attn_out=attn_out, outputs=e_outs, ws=ws)
             if host_clock:
                 api_s[0] += time.perf_counter() - t0
-            for hd, dd in zip(h_out[k], outs[:3]):
-                hd.copy_(dd, non_blocking=True)
-            free[k] = torch.cuda.Event()
-            free[k].record(stream)
+            h_out[k].copy_(d_out, non_blocking=True)
+            ev_free[k].record(stream)
         stream.wait_stream(cs)
 
     # plain calls: the library's host work (validation, planning, launches)
@@ -609,8 +631,9 @@ def write_line(args, b, world, hbm_peak, peak_kind, stages, total_ms_max, units_
                 "unit": "verified tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": e2e_max / n_steps, "api_host_us_per_call": api_us,
                 "schedule": "plain calls through the Python API (the library's validation and planning included); "
-                            "per step: pinned H2D of q, logits, drafts on a copy stream; the call; D2H of "
-                            "accept_len, offsets, tokens; uploads overlap the previous step's compute; host clock"},
+                            "per step: one pinned H2D copy of q, logits and drafts (packed) on a copy stream; "
+                            "the call; one D2H copy of accept_len, offsets, tokens (packed); uploads overlap "
+                            "the previous step's compute; host clock"},
         "e2e_graph": {"value": emitted / (e2e_graph_ms / 1000.0), "unit": "verified tokens/s",
                       "ms_per_step": e2e_graph_ms,
                       "schedule": "the same steps captured as one CUDA graph of the API calls, replayed back to back"},

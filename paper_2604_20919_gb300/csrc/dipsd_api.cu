@@ -222,7 +222,17 @@ static std::vector<int> cut_chunks(const std::vector<int>& np, int grid) {
   };
   long long total = 0;
   for (int pages : np) total += pages + kPiecePages;
-  long long lo = 1, hi = total + kPiecePages;  // cut(hi) gives one chunk
+  // Every chunk carries at most `cap`, so the smallest feasible cap is at
+  // least total / grid; every chunk but the last carries at least cap minus
+  // one piece's charge of the streams' own cost, and each cut adds one piece
+  // charge, so total / grid + 2 kPiecePages is feasible.  Search that narrow
+  // range first; the whole range only if it fails.
+  long long lo = std::max<long long>(1, total / std::max(1, grid));
+  long long hi = lo + 4 * kPiecePages + 64;
+  if (cut(hi, nullptr) > grid) {
+    lo = hi + 1;
+    hi = total + kPiecePages;  // cut(hi) gives one chunk
+  }
   while (lo < hi) {
     const long long mid = (lo + hi) / 2;
     if (cut(mid, nullptr) <= grid) hi = mid; else lo = mid + 1;

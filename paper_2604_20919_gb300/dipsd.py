@@ -44,7 +44,7 @@ TEST_OVERRIDES = {"attn_split_tiles": 1, "attn_cluster": 2, "attn_persist": 3, "
                   "spec_nk1": 5, "spec_nk2": 6}
 
 _lib: Optional[ctypes.CDLL] = None
-_i32p = ctypes.POINTER(ctypes.c_int)
+_i32p = ctypes.c_void_p  # host int32 arrays, passed by address
 _vp = ctypes.c_void_p
 _sz = ctypes.c_size_t
 _i = ctypes.c_int
@@ -148,18 +148,22 @@ def _check(status: int, where: str) -> None:
 
 
 def _host_i32(x: Sequence[int]):
-    a = np.ascontiguousarray(np.asarray(x, dtype=np.int32))
-    return a, a.ctypes.data_as(_i32p)
+    """A C-contiguous int32 host array of x (x itself when it already is one)
+    and its address; the array must outlive the call that gets the address."""
+    if type(x) is np.ndarray and x.dtype == np.int32 and x.flags.c_contiguous:
+        a = x
+    else:
+        a = np.ascontiguousarray(x, dtype=np.int32)
+    return a, a.ctypes.data
 
 
 def _dptr(t: Optional[torch.Tensor], name: str, dtype=None) -> int:
+    """Device address of a contiguous CUDA tensor (of dtype, if given)."""
     if t is None:
         return 0
-    if not t.is_cuda:
-        raise ValueError(f"{name} must be a CUDA tensor")
-    if not t.is_contiguous():
-        raise ValueError(f"{name} must be contiguous")
-    if dtype is not None and t.dtype != dtype:
+    if not (t.is_cuda and t.is_contiguous()):
+        raise ValueError(f"{name} must be a contiguous CUDA tensor")
+    if dtype is not None and t.dtype is not dtype:
         raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
     return t.data_ptr()
 
@@ -394,21 +398,21 @@ def _verify_batch(members, L_all, ctx_all, q, k_cache, v_cache, block_table_all,
 
     Returns (attn_out, accept_len, out_offsets, out_tokens, draft_probs).
     """
-    lib = load()
+    lib = _lib if _lib is not None else load()
     m, pm = _host_i32(members)
     a, pa = _host_i32(L_all)
     b, pb = _host_i32(ctx_all)
-    Lb = a[m]
-    sum_t, sum_l = int((Lb + 1).sum()), int(Lb.sum())
+    sum_l = int(a[m].sum())  # (a member outside the tables raises IndexError here)
+    sum_t = sum_l + len(m)
     nb, Hkv, page, D = k_cache.shape
     Hq, V = q.shape[1], target_logits.shape[1]
-    if page != PAGE_SIZE or tuple(q.shape) != (sum_t, Hq, D):
+    if page != PAGE_SIZE or q.shape != (sum_t, Hq, D):
         raise ValueError("q does not match the members' draft lengths")
     if target_logits.shape[0] != sum_t or draft_logits.shape != (sum_l, V):
         raise ValueError("logits do not match the members' draft lengths")
     if attn_out is None:
         attn_out = torch.empty_like(q)
-    acc, offs, toks, probs = outputs if outputs is not None else spec_outputs(Lb, q.device)
+    acc, offs, toks, probs = outputs if outputs is not None else spec_outputs(a[m], q.device)
     if ws is None:
         ws = workspace(dipsd_verify_batch_workspace_size(m, a, b, Hq, Hkv, D, V), q.device)
     if new_kv is not None:
