@@ -367,6 +367,8 @@ int dipsd_verify_uniforms(int B, const int* h_L, const int* h_user_id, uint64_t 
  *   DIPSD_TEST_SPEC_NK1,
  *   DIPSD_TEST_SPEC_NK2          16-byte vectors per lane in a segment of the
  *                                two sampling passes (one of 16/8/4, 8/4/2)
+ *   DIPSD_TEST_SPEC_GRID1        at most this many CTAs in the statistics
+ *                                pass, so each warp takes several segments
  * Returns DIPSD_ERR_INVALID_ARG for an unknown code or a negative value.
  * ---------------------------------------------------------------------- */
 #define DIPSD_TEST_ATTN_SPLIT_TILES 1
@@ -375,6 +377,7 @@ int dipsd_verify_uniforms(int B, const int* h_L, const int* h_user_id, uint64_t 
 #define DIPSD_TEST_ATTN_GRID 4
 #define DIPSD_TEST_SPEC_NK1 5
 #define DIPSD_TEST_SPEC_NK2 6
+#define DIPSD_TEST_SPEC_GRID1 7
 int dipsd_test_set_override(int which, int value);
 
 #ifdef __cplusplus

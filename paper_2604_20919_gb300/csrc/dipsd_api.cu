@@ -33,7 +33,7 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Plan overrides set through dipsd_test_set_override (0 = the planner's own
 // choice); indexed by the DIPSD_TEST_* codes of dipsd.h.
-constexpr int kNumOverrides = 7;
+constexpr int kNumOverrides = 8;
 std::atomic<int> g_override[kNumOverrides];
 int plan_override(int which) { return g_override[which].load(std::memory_order_relaxed); }
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
@@ -520,6 +520,7 @@ int check_attn_buffers(const void* q, const void* kc, const void* vc, int num_bl
 struct SpecPlan {
   int B = 0, V = 0, vec = 1, nvec = 0, cl1 = 1, cl2 = 1;
   int nk1 = 0, nk2 = 0;  // register path: vectors per lane and segment (0 = generic path)
+  int grid1 = 0;         // register path: CTAs of the (persistent) statistics pass
   int nseg1 = 0, nseg2 = 0, n_items1 = 0, n_items2 = 0;
   int sum_t = 0, sum_l = 0;
   bool sparse = false;  // sparse draft payload: no draft logit rows
@@ -577,7 +578,7 @@ void plan_spec(int B, const int* L, int V, int elem, bool vec_ok, int sms, SpecP
   }
   pl.sum_t = pl.q_off[B];
   pl.sum_l = pl.l_off[B];
-  pl.nk1 = pl.nk2 = 0;
+  pl.nk1 = pl.nk2 = pl.grid1 = 0;
   pl.nseg1 = pl.nseg2 = pl.n_items1 = pl.n_items2 = 0;
   size_t o = align_up(static_cast<size_t>(pl.sum_t) * sizeof(SpecStat), 256);
   pl.off_flags = o;
@@ -603,6 +604,11 @@ void plan_spec(int B, const int* L, int V, int elem, bool vec_ok, int sms, SpecP
       o += align_up(static_cast<size_t>(items1) * sizeof(float4), 256);
       pl.off_part2 = o;
       o += align_up(static_cast<size_t>(items2) * sizeof(float4), 256);
+      // statistics pass: two resident CTAs per SM at most, each warp taking
+      // several segments in turn when there are more (or a test's cap)
+      pl.grid1 = ceil_div(pl.n_items1, kRegWarps);
+      if (sms > 0) pl.grid1 = std::min(pl.grid1, 2 * sms);
+      if (const int v = plan_override(DIPSD_TEST_SPEC_GRID1)) pl.grid1 = std::min(pl.grid1, v);
     }
   }
   pl.ws_bytes = o;
@@ -659,8 +665,11 @@ int launch_spec_sample_t(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStrea
 
 template <typename T, int NK1, int CAP, bool SP>
 int launch_spec_reg_t(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s, bool pdl) {
-  if (launch(spec_stats_kernel<T, NK1, CAP, SP>, dim3(ceil_div(pl.n_items1, kRegWarps)), dim3(kRegThreads), 0, s, 1,
-             pdl, p) != cudaSuccess)
+  if (launch(spec_stats_kernel<T, NK1, CAP, SP>, dim3(pl.grid1), dim3(kRegThreads), 0, s, 0, pdl, p) !=
+      cudaSuccess)
+    return DIPSD_ERR_CUDA;
+  if (launch(spec_decide_kernel<CAP, SP>, dim3(ceil_div(pl.sum_t, kRegWarps)), dim3(kRegThreads), 0, s, 0, true,
+             p) != cudaSuccess)
     return DIPSD_ERR_CUDA;
   if constexpr (SP) {  // the table's q of every element stays in registers: at most 4 vectors per lane
     return pl.nk2 == 4 ? launch_spec_sample_t<T, 4, CAP, SP>(pl, p, s) : launch_spec_sample_t<T, 2, CAP, SP>(pl, p, s);

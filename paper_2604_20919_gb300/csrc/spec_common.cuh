@@ -13,11 +13,10 @@ constexpr int kSpecWarps = kSpecThreads / 32;
 constexpr int kMaxCluster = 8;
 constexpr unsigned kDevErrBadToken = 2u;
 constexpr int kMaxTopK = 64;  // sparse payload: table entries per draft row
-// Arrival counters of the register path, in 32-bit words: one per verify
-// position; then one 64-bit word per user for the decisions (arrivals in the
-// high half, acceptance bit t of position t in the low half); then one per
-// user for the sampling segments.
-constexpr int kCntUser1 = kMaxUsers * (kMaxDraft + 1);
+// Counters of the register path, in 32-bit words: one 64-bit word per user
+// for the decisions (arrivals in the high half, acceptance bit t of position
+// t in the low half); then one per user for the sampling segments.
+constexpr int kCntUser1 = 0;
 constexpr int kCntUser2 = kCntUser1 + 2 * kMaxUsers;
 constexpr int kCounterWords = kCntUser2 + kMaxUsers;
 

@@ -3,31 +3,32 @@
 // rejection, emit one more token from the residual or, at the bonus position,
 // from the target distribution).  Register path for 16-byte aligned rows.
 //
-// Both kernels are flat over warps.  A work item is one warp-sized segment of
-// one row: 32 lanes x NK 16-byte vectors, lane-interleaved so that every load
-// instruction of the warp reads 512 contiguous bytes, all of a lane's loads
-// issued before the first use.  Items spread evenly over the SMs whatever the
-// mix of draft lengths.  Segments meet through arrival counters in global
-// memory: the warp that delivers the last segment of a position (or of a
-// user) goes on with the step that needs them all, and no warp ever waits for
-// another.
+// Three kernels, chained by programmatic dependent launch.  A work item of
+// the two streaming passes is one warp-sized segment of one row: 32 lanes x
+// NK 16-byte vectors, lane-interleaved so that every load instruction of the
+// warp reads 512 contiguous bytes.  Items spread evenly over the SMs whatever
+// the mix of draft lengths.
 //
-// spec_stats_kernel: items are the segments of every target row z_t and every
-// draft row w_t.  A warp takes the integer reference c = ceil(m log2 e) of its
-// segment maximum m and sums 2^(x log2 e - c) (two FFMA and one ex2 per
-// logit).  References are integers, so partial sums combine by exact
-// power-of-two rescaling as float-float pairs.  The last segment of position
-// t combines the row sums, forms p_t(d), q_t(d) and decides
-// u_acc * q_t(d) < p_t(d); the last decided position of user i counts the
-// leading accepts a_i.
+// spec_stats_kernel: the segments of every target row z_t and every draft row
+// w_t, persistent over warps.  A warp takes the integer reference
+// c = ceil(m log2 e) of a group's maximum m and sums 2^(x log2 e - c) (two
+// FFMA and one ex2 per logit).  References are integers, so partial sums
+// combine by exact power-of-two rescaling as float-float pairs.  Each segment
+// leaves its partial; no atomics, no waits.
 //
-// spec_sample_kernel: items are the segments of the rows at position a_i of
-// every user.  A warp computes the sampling weights (max(0, p - q) up to a
-// common factor, or p at the bonus position) and stores its segment's total,
-// summed in token order: fp32 scans over 32-vector groups, float-float across
-// groups.  The last segment of user i locates u * total: segment, group, lane
-// and token, replaying the very sums that produced the totals, so the descent
-// lands in the cell the totals point to.
+// spec_decide_kernel: one warp per position combines its rows' partials,
+// forms p_t(d), q_t(d) and decides u_acc * q_t(d) < p_t(d); the last decided
+// position of user i (a 64-bit decision word per user) counts the leading
+// accepts a_i.
+//
+// spec_sample_kernel: the segments of the rows at position a_i of every
+// user.  A warp computes the sampling weights (max(0, p - q) up to a common
+// factor, or p at the bonus position) and stores its segment's total, summed
+// in token order: fp32 scans over 32-vector groups, float-float across
+// groups.  The warp that delivers the last segment of user i (an arrival
+// counter) locates u * total: segment, group, lane and token, replaying the
+// very sums that produced the totals, so the descent lands in the cell the
+// totals point to.
 #pragma once
 
 #include "spec_common.cuh"
@@ -569,9 +570,8 @@ __device__ __forceinline__ void decide_from_sums(const SpecParams<CAP>& p, int u
   }
 }
 
-// Run by the warp that delivered the last segment of position q0 + t of user
-// ui: row sums, p_t(d), q_t(d), the acceptance decision; the user's last
-// decided position also writes a_i.
+// Row sums, p_t(d), q_t(d) and the acceptance decision of position q0 + t of
+// user ui (one warp); the user's last decided position also writes a_i.
 template <int CAP, bool SP>
 __device__ __forceinline__ void decide_position(const SpecParams<CAP>& p, int ui, int t, int lane) {
   const int q0 = p.q_off[ui];
@@ -600,64 +600,120 @@ __device__ __forceinline__ void decide_position(const SpecParams<CAP>& p, int ui
   }
   az = warp_refsum(az);
   if (has_q && !SP) aw = warp_refsum(aw);
-  if (lane == 0) {
-    p.counters[n] = 0u;
-    decide_from_sums<CAP, SP>(p, ui, t, az, aw, zd, wd, logq, u_acc);
-  }
+  if (lane == 0) decide_from_sums<CAP, SP>(p, ui, t, az, aw, zd, wd, logq, u_acc);
 }
 
 // ------------------------------------------------------------------ pass 1
+// One segment of one logit row: z_t of user ui, or w_t.
+template <typename T>
+struct StatSeg {
+  const T* row;
+  int item, vb, nv, l;
+  bool has_q;
+};
+
+// Segment `item` of the flat item list (rows: every z_t, then every w_t; no
+// w rows when the draft payload is sparse).
+template <typename T, int NK, int CAP, bool SP>
+__device__ __forceinline__ StatSeg<T> stat_seg(const SpecParams<CAP>& p, int item, int lane) {
+  const int row = item / p.nseg1;
+  const int s = item - row * p.nseg1;
+  const bool is_w = !SP && row >= p.sum_t;
+  const int ui = is_w ? spec_find_user<CAP>(p.l_off, p.B, row - p.sum_t) : spec_find_user<CAP>(p.q_off, p.B, row);
+  const int q0 = p.q_off[ui];
+  const int t = is_w ? row - p.sum_t - p.l_off[ui] : row - q0;
+  StatSeg<T> g;
+  g.item = item;
+  g.l = p.l_off[ui] + t;
+  g.has_q = t < p.q_off[ui + 1] - q0 - 1;
+  g.row = is_w ? static_cast<const T*>(p.w) + static_cast<size_t>(g.l) * p.V
+               : static_cast<const T*>(p.z) + static_cast<size_t>(q0 + t) * p.V;
+  g.vb = s * (32 * NK);
+  g.nv = lane_vectors(p.nvec, g.vb, lane, NK);
+  return g;
+}
+
+// The draft token's logit in the row, fetched by lane 0 of the row's first
+// segment (NaN: the token lies outside [0, V)); 0 elsewhere.
+template <typename T, int CAP>
+__device__ __forceinline__ float stat_draft_logit(const SpecParams<CAP>& p, const StatSeg<T>& g, int lane) {
+  if (g.vb != 0 || lane != 0 || !g.has_q) return 0.f;
+  const int d = p.draft_tokens[g.l];
+  return d >= 0 && d < p.V ? load_elem<T>(g.row, d) : __int_as_float(0x7fc00000);
+}
+
+// Loads a lane's vectors k0 .. k0 + KG - 1 of a segment (zero past nv).
+template <int NK, int KG>
+__device__ __forceinline__ void load_group(const void* row, int vb, int lane, int nv, int k0, uint4 (&r)[NK]) {
+  const uint8_t* q = static_cast<const uint8_t*>(row) + (static_cast<size_t>(vb) + lane) * 16;
+#pragma unroll
+  for (int k = k0; k < k0 + KG; ++k)
+    r[k] = k < nv ? ldg_stream_v4(q + static_cast<size_t>(k) * 512) : make_uint4(0u, 0u, 0u, 0u);
+}
+
+// Row sums of every segment, persistent over warps: warp w of the W in the
+// grid takes items w, w + W, w + 2W, ...  A segment's vectors go in groups of
+// four, each group with its own warp reference, so the first group's
+// exponentials overlap the later groups' loads; once a group is summed its
+// registers are refilled with the same group of the warp's next segment, so
+// the warp keeps about one segment of loads in flight from its first segment
+// to its last.  Each segment's partial (reference, float-float sum, draft
+// logit) goes to part1; no warp waits for another, and nothing here orders
+// the partials: the decision kernel reads them once this grid is complete.
 template <typename T, int NK, int CAP, bool SP>
 __global__ void __launch_bounds__(kRegThreads, 2)
 spec_stats_kernel(const __grid_constant__ SpecParams<CAP> p) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int item = blockIdx.x * kRegWarps + warp;
+  const int lane = threadIdx.x & 31;
+  const int W = gridDim.x * kRegWarps;
+  int item = blockIdx.x * kRegWarps + (threadIdx.x >> 5);
   pdl_wait_prior_grid();
   pdl_launch_dependents();
   if (item >= p.n_items1) return;
-  const int row = item / p.nseg1;
-  const int s = item - row * p.nseg1;
-  const bool is_w = !SP && row >= p.sum_t;  // rows: every z_t, then every w_t (none when sparse)
-  const int ui = is_w ? spec_find_user<CAP>(p.l_off, p.B, row - p.sum_t) : spec_find_user<CAP>(p.q_off, p.B, row);
-  const int q0 = p.q_off[ui];
-  const int Li = p.q_off[ui + 1] - q0 - 1;
-  const int t = is_w ? row - p.sum_t - p.l_off[ui] : row - q0;
-  const int n = q0 + t, l = p.l_off[ui] + t;
-  const bool has_q = t < Li;
-  const T* rowp = is_w ? static_cast<const T*>(p.w) + static_cast<size_t>(l) * p.V
-                       : static_cast<const T*>(p.z) + static_cast<size_t>(n) * p.V;
-  const int vb = s * (32 * NK);
-  const int nv = lane_vectors(p.nvec, vb, lane, NK);
-  uint4 r[NK];
-  load_segment<NK>(rowp, vb, lane, nv, r);
-  // the draft token's logit, fetched by lane 0 of the row's first segment
-  float xd = 0.f;
-  if (s == 0 && lane == 0 && has_q) {
-    const int d = p.draft_tokens[l];
-    xd = d >= 0 && d < p.V ? load_elem<T>(rowp, d) : __int_as_float(0x7fc00000);
-  }
-  // groups of four vectors, each with its own warp reference, so that the
-  // first group's exponentials overlap the later groups' loads
   constexpr int KG = NK < 4 ? NK : 4;
-  RefSum tot{kEmptyRef, FF{0.f, 0.f}};
+  StatSeg<T> g = stat_seg<T, NK, CAP, SP>(p, item, lane);
+  uint4 r[NK];
+  load_segment<NK>(g.row, g.vb, lane, g.nv, r);
+  float xd = stat_draft_logit<T, CAP>(p, g, lane);
+  for (;;) {
+    const int nxt = item + W;
+    const bool more = nxt < p.n_items1;
+    StatSeg<T> ng = g;
+    float nxd = 0.f;
+    if (more) {
+      ng = stat_seg<T, NK, CAP, SP>(p, nxt, lane);
+      nxd = stat_draft_logit<T, CAP>(p, ng, lane);
+    }
+    RefSum tot{kEmptyRef, FF{0.f, 0.f}};
 #pragma unroll
-  for (int k0 = 0; k0 < NK; k0 += KG) {
-    const float m = lane_max<T, NK, KG>(r, k0, nv);
-    int c = m > -INFINITY ? static_cast<int>(fminf(fmaxf(ceilf(m * kLog2e), -1048576.f), 1048576.f)) : kEmptyRef;
-    c = __reduce_max_sync(0xffffffffu, c);
-    if (c != kEmptyRef) tot = refsum_add(tot, RefSum{c, lane_expsum<T, NK, KG>(r, k0, nv, static_cast<float>(c))});
+    for (int k0 = 0; k0 < NK; k0 += KG) {
+      const float m = lane_max<T, NK, KG>(r, k0, g.nv);
+      int c = m > -INFINITY ? static_cast<int>(fminf(fmaxf(ceilf(m * kLog2e), -1048576.f), 1048576.f)) : kEmptyRef;
+      c = __reduce_max_sync(0xffffffffu, c);
+      if (c != kEmptyRef) tot = refsum_add(tot, RefSum{c, lane_expsum<T, NK, KG>(r, k0, g.nv, static_cast<float>(c))});
+      if (more) load_group<NK, KG>(ng.row, ng.vb, lane, ng.nv, k0, r);
+    }
+    const FF sum = warp_ff_sum(tot.s);
+    if (lane == 0) p.part1[g.item] = make_float4(__int_as_float(tot.c), sum.hi, sum.lo, xd);
+    if (!more) break;
+    item = nxt;
+    g = ng;
+    xd = nxd;
   }
-  const int c = tot.c;  // the same in every lane
-  const FF sum = warp_ff_sum(tot.s);
-  unsigned cnt = 0;
-  if (lane == 0) {
-    p.part1[item] = make_float4(__int_as_float(c), sum.hi, sum.lo, xd);
-    cnt = counter_arrive(p.counters + n);
-  }
-  __syncwarp();
-  cnt = __shfl_sync(0xffffffffu, cnt, 0);
-  if (cnt != static_cast<unsigned>(p.nseg1 * (has_q && !SP ? 2 : 1))) return;
-  decide_position<CAP, SP>(p, ui, t, lane);
+}
+
+// One warp per verify position: the row sums from the statistics pass's
+// partials, p_t(d), q_t(d) and the acceptance decision; the user's last
+// decided position writes a_i.
+template <int CAP, bool SP>
+__global__ void __launch_bounds__(kRegThreads)
+spec_decide_kernel(const __grid_constant__ SpecParams<CAP> p) {
+  const int lane = threadIdx.x & 31;
+  const int n = blockIdx.x * kRegWarps + (threadIdx.x >> 5);
+  pdl_wait_prior_grid();
+  pdl_launch_dependents();
+  if (n >= p.sum_t) return;
+  const int ui = spec_find_user<CAP>(p.q_off, p.B, n);
+  decide_position<CAP, SP>(p, ui, n - p.q_off[ui], lane);
 }
 
 // ------------------------------------------------------------------ pass 2

@@ -164,3 +164,24 @@ def test_spec_verify_segment_sizes(cuda_lib, nk1, nk2):
     with cuda_lib.plan_override(spec_nk1=nk1, spec_nk2=nk2):
         st = check_spec(b, *_run(cuda_lib, b))
     print(f"segments {nk1}/{nk2}: {st}")
+
+
+@pytest.mark.parametrize("grid1,nk1", [(1, 16), (3, 8), (40, 4), (97, 16)])
+def test_spec_verify_persistent_statistics_grid(cuda_lib, grid1, nk1):
+    """The statistics pass on a capped grid, so every warp sums many segments
+    in turn (each refilled while the previous one is summed); three calls in a
+    row, so the decision words and arrival counters must come back to zero."""
+    rng = np.random.default_rng(50 + grid1)
+    L = np.concatenate([[0, 31, 0], rng.integers(0, 11, size=37)])
+    b = make_batch(L, np.zeros_like(L), Hq=8, Hkv=1, D=64, V=30016, logit_std=2.0, noise_sigma=0.8,
+                   seed=50 + grid1, spec_only=True)
+    g = lambda t: t.to(DEV)
+    ws = cuda_lib.workspace(cuda_lib.dipsd_spec_verify_workspace_size(b.L, b.V), DEV)
+    with cuda_lib.plan_override(spec_grid1=grid1, spec_nk1=nk1):
+        for _ in range(3):
+            out = cuda_lib.dipsd_spec_verify(b.L, b.user_ids, b.seed, g(b.target_logits), g(b.draft_logits),
+                                             g(b.draft_tokens), ws=ws)
+            torch.cuda.synchronize()
+            st = check_spec(b, *out)
+            assert cuda_lib.device_status(ws) == 0
+    print(f"statistics grid {grid1} x {nk1}: {st}")
