@@ -525,7 +525,7 @@ struct SpecPlan {
   int sum_t = 0, sum_l = 0;
   bool sparse = false;  // sparse draft payload: no draft logit rows
   std::vector<int> q_off, l_off;
-  size_t off_flags = 0, off_part1 = 0, off_part2 = 0;
+  size_t off_flags = 0, off_ures = 0, off_part1 = 0, off_part2 = 0;
   size_t ws_bytes = 0;  // spec region only
 };
 
@@ -583,6 +583,8 @@ void plan_spec(int B, const int* L, int V, int elem, bool vec_ok, int sms, SpecP
   size_t o = align_up(static_cast<size_t>(pl.sum_t) * sizeof(SpecStat), 256);
   pl.off_flags = o;
   o += align_up(pl.sum_t, 256);
+  pl.off_ures = o;
+  o += align_up(static_cast<size_t>(pl.sum_t) * sizeof(float), 256);
   pl.off_part1 = pl.off_part2 = o;
   if (vec_ok) {
     const int rows = pl.sum_t + (sparse ? 0 : pl.sum_l);
@@ -710,6 +712,7 @@ int run_spec_cap(const SpecPlan& pl, int dtype, const void* z, const void* w, co
   for (int i = 0; i < pl.B; ++i) p.uid[i] = uid[i];
   p.stats = region;
   p.flags = region + pl.off_flags;
+  p.u_res = reinterpret_cast<float*>(region + pl.off_ures);
   p.part1 = reinterpret_cast<float4*>(region + pl.off_part1);
   p.part2 = reinterpret_cast<float4*>(region + pl.off_part2);
   p.counters = reinterpret_cast<unsigned*>(reinterpret_cast<uint8_t*>(status) + kStatusBytes);

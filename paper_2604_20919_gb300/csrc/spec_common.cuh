@@ -27,6 +27,7 @@ struct SpecParams {
   const int* draft_tokens;    // [sum L]
   void* stats;                // [sum T] row statistics (layout private to each path)
   unsigned char* flags;       // [sum T]: acceptance bit
+  float* u_res;               // [sum T]: resample uniform of each position (register path)
   float* draft_probs;         // optional [sum T][2]
   int* accept_len;            // [B]
   int* out_offsets;           // [B+1]

@@ -589,8 +589,11 @@ __device__ __forceinline__ void decide_position(const SpecParams<CAP>& p, int ui
     else wd = __ldcg(&pw->w);
   }
   RefSum az{kEmptyRef, FF{0.f, 0.f}}, aw{kEmptyRef, FF{0.f, 0.f}};
-  // the acceptance uniform (independent of the loads, so it overlaps them)
-  const float u_acc = has_q ? verify_uniforms(p.seed, static_cast<unsigned>(p.uid[ui]), t).x : 0.f;
+  // the position's two uniforms (independent of the loads, so they overlap
+  // them): the acceptance one here, the resample one kept for the descent
+  const float2 u = verify_uniforms(p.seed, static_cast<unsigned>(p.uid[ui]), t);
+  const float u_acc = has_q ? u.x : 0.f;
+  if (lane == 0) p.u_res[n] = u.y;
 #pragma unroll 2
   for (int sg = lane; sg < p.nseg1; sg += 32) {
     const float4 vz = __ldcg(pz + sg);
@@ -746,7 +749,7 @@ __device__ __forceinline__ void descend(const SpecParams<CAP>& p, int ui, int a,
   const int mode0 = residual ? 0 : 1;
   float2 v[kRun];
   load_run(mode0, v);
-  const float u = verify_uniforms(p.seed, static_cast<unsigned>(p.uid[ui]), a).y;
+  const float u = __ldcg(p.u_res + p.q_off[ui] + a);  // drawn by the decision kernel
   const int dtok = lane < a ? p.draft_tokens[l0 + lane] : 0;  // a <= L_i <= 31
   int o = 0;
   for (int j = lane; j < ui; j += 32)
