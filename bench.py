@@ -291,7 +291,9 @@ def capture(fn, n, R, stream):
     stream.wait_stream(side)
     torch.cuda.synchronize()
     n0 = dipsd.dipsd_launch_count()
-    with torch.cuda.graph(g):
+    # captured on the stream that made the warm-up calls: the library's
+    # per-stream resources (verify_batch's second stream) exist by then
+    with torch.cuda.graph(g, stream=side):
         for i in range(n):
             fn(i)
     torch.cuda.synchronize()
@@ -521,7 +523,8 @@ def run_dipsd(args):
     api_s = [0.0]
 
     def e2e_steps(n, host_clock=False):
-        cs.wait_stream(stream)
+        cur = torch.cuda.current_stream()  # the compute stream (a capture's stream inside one)
+        cs.wait_stream(cur)
         for i in range(n):
             k = i % R
             c = e_in[k]
@@ -530,15 +533,16 @@ def run_dipsd(args):
             with torch.cuda.stream(cs):
                 d_in[k].copy_(h_in, non_blocking=True)
             ev_up[k].record(cs)
-            stream.wait_event(ev_up[k])
+            cur.wait_event(ev_up[k])
             t0 = time.perf_counter()
             dipsd.dipsd_verify_batch(b.members, b.L, b.ctx, c["q"], copies[k]["kc"], copies[k]["vc"], bt, b.scale,
-                                     c["z"], c["w"], c["d"], b.seed, attn_out=attn_out, outputs=e_outs, ws=ws)
+                                     c["z"], c["w"], c["d"], b.seed, attn_out=attn_out, outputs=e_outs, ws=ws,
+                                     stream=cur)
             if host_clock:
                 api_s[0] += time.perf_counter() - t0
             h_out[k].copy_(d_out, non_blocking=True)
-            ev_free[k].record(stream)
-        stream.wait_stream(cs)
+            ev_free[k].record(cur)
+        cur.wait_stream(cs)
 
     # plain calls: the library's host work (validation, planning, launches)
     # and the binding's argument marshalling are inside the timed region
@@ -551,9 +555,15 @@ def run_dipsd(args):
     torch.cuda.synchronize()
     e2e_plain_ms = 1000 * (time.perf_counter() - t0) / n_steps
     api_us = 1e6 * api_s[0] / n_steps
-    # the same steps captured as one CUDA graph, replayed back to back
+    # the same steps captured as one CUDA graph, replayed back to back (on a
+    # stream that made plain calls first)
     g_e2e = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g_e2e):
+    cap = torch.cuda.Stream()
+    cap.wait_stream(stream)
+    with torch.cuda.stream(cap):
+        e2e_steps(R)
+    torch.cuda.synchronize()
+    with torch.cuda.graph(g_e2e, stream=cap):
         e2e_steps(R)
     g_e2e.replay()
     torch.cuda.synchronize()

@@ -238,10 +238,15 @@ int dipsd_spec_verify_sparse(int B, const int* h_L, const int* h_user_id, uint64
 
 /* ------------------------------------------------------------------------
  * One pipeline stage: the users of batch n (Sec. III-C, B_n(x)) verified
- * together -- attention and speculative verification, on one stream.  The
- * two stages read disjoint inputs and run overlapped (the attention grid
- * streams the KV cache while the sampling kernel finishes); all outputs are
- * complete when the work queued on the stream completes.  No output buffer
+ * together -- attention and speculative verification.  The two stages read
+ * disjoint inputs and run overlapped: after the statistics pass of the
+ * speculative verification, the attention grid runs on `stream` while the
+ * decision and sampling kernels run beside it on a second stream that the
+ * library keeps per host thread, device and caller stream (made on the first
+ * call from that thread and stream outside a stream capture; it lives until
+ * the thread exits) and joins back into `stream` before the call returns.
+ * All outputs are complete when the work queued on `stream` completes; a
+ * call captured into a CUDA graph captures both streams.  No output buffer
  * may overlap an input buffer.
  *
  * Per-user tables cover all M users being served; h_members[b] (distinct, in
@@ -369,6 +374,9 @@ int dipsd_verify_uniforms(int B, const int* h_L, const int* h_user_id, uint64_t 
  *                                two sampling passes (one of 16/8/4, 8/4/2)
  *   DIPSD_TEST_SPEC_GRID1        at most this many CTAs in the statistics
  *                                pass, so each warp takes several segments
+ *   DIPSD_TEST_BATCH_FORK        verify_batch: 1 = decision and sampling on a
+ *                                second stream beside the attention grid (the
+ *                                default), 2 = everything on the one stream
  * Returns DIPSD_ERR_INVALID_ARG for an unknown code or a negative value.
  * ---------------------------------------------------------------------- */
 #define DIPSD_TEST_ATTN_SPLIT_TILES 1
@@ -378,6 +386,7 @@ int dipsd_verify_uniforms(int B, const int* h_L, const int* h_user_id, uint64_t 
 #define DIPSD_TEST_SPEC_NK1 5
 #define DIPSD_TEST_SPEC_NK2 6
 #define DIPSD_TEST_SPEC_GRID1 7
+#define DIPSD_TEST_BATCH_FORK 8
 int dipsd_test_set_override(int which, int value);
 
 #ifdef __cplusplus

@@ -33,7 +33,7 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Plan overrides set through dipsd_test_set_override (0 = the planner's own
 // choice); indexed by the DIPSD_TEST_* codes of dipsd.h.
-constexpr int kNumOverrides = 8;
+constexpr int kNumOverrides = 9;
 std::atomic<int> g_override[kNumOverrides];
 int plan_override(int which) { return g_override[which].load(std::memory_order_relaxed); }
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
@@ -665,13 +665,28 @@ int launch_spec_sample_t(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStrea
                 s, 1, true, p) == cudaSuccess ? DIPSD_OK : DIPSD_ERR_CUDA;
 }
 
+// A second stream the decision and sampling kernels may move to after the
+// statistics pass (aux null: everything on the caller's stream).
+struct SpecFork {
+  cudaStream_t aux = nullptr;
+  cudaEvent_t fork = nullptr;
+};
+
 template <typename T, int NK1, int CAP, bool SP>
-int launch_spec_reg_t(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s, bool pdl) {
+int launch_spec_reg_t(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s, bool pdl,
+                      const SpecFork& fk) {
   if (launch(spec_stats_kernel<T, NK1, CAP, SP>, dim3(pl.grid1), dim3(kRegThreads), 0, s, 0, pdl, p) !=
       cudaSuccess)
     return DIPSD_ERR_CUDA;
-  if (launch(spec_decide_kernel<CAP, SP>, dim3(ceil_div(pl.sum_t, kRegWarps)), dim3(kRegThreads), 0, s, 0, true,
-             p) != cudaSuccess)
+  bool pdl_decide = true;
+  if (fk.aux) {  // the rest of the stage behind the statistics pass, on the second stream
+    if (cudaEventRecord(fk.fork, s) != cudaSuccess || cudaStreamWaitEvent(fk.aux, fk.fork, 0) != cudaSuccess)
+      return DIPSD_ERR_CUDA;
+    s = fk.aux;
+    pdl_decide = false;
+  }
+  if (launch(spec_decide_kernel<CAP, SP>, dim3(ceil_div(pl.sum_t, kRegWarps)), dim3(kRegThreads), 0, s, 0,
+             pdl_decide, p) != cudaSuccess)
     return DIPSD_ERR_CUDA;
   if constexpr (SP) {  // the table's q of every element stays in registers: at most 4 vectors per lane
     return pl.nk2 == 4 ? launch_spec_sample_t<T, 4, CAP, SP>(pl, p, s) : launch_spec_sample_t<T, 2, CAP, SP>(pl, p, s);
@@ -685,11 +700,11 @@ int launch_spec_reg_t(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t
 }
 
 template <typename T, int CAP, bool SP>
-int launch_spec_reg(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s, bool pdl) {
+int launch_spec_reg(const SpecPlan& pl, const SpecParams<CAP>& p, cudaStream_t s, bool pdl, const SpecFork& fk) {
   switch (pl.nk1) {
-    case 16: return launch_spec_reg_t<T, 16, CAP, SP>(pl, p, s, pdl);
-    case 8: return launch_spec_reg_t<T, 8, CAP, SP>(pl, p, s, pdl);
-    default: return launch_spec_reg_t<T, 4, CAP, SP>(pl, p, s, pdl);
+    case 16: return launch_spec_reg_t<T, 16, CAP, SP>(pl, p, s, pdl, fk);
+    case 8: return launch_spec_reg_t<T, 8, CAP, SP>(pl, p, s, pdl, fk);
+    default: return launch_spec_reg_t<T, 4, CAP, SP>(pl, p, s, pdl, fk);
   }
 }
 
@@ -704,7 +719,7 @@ struct SparseDraft {
 template <int CAP>
 int run_spec_cap(const SpecPlan& pl, int dtype, const void* z, const void* w, const int* dt, uint64_t seed,
                  const int* uid, int* acc, int* offs, int* toks, float* probs, unsigned* status, uint8_t* region,
-                 cudaStream_t s, bool pdl, const SparseDraft& sd) {
+                 cudaStream_t s, bool pdl, const SparseDraft& sd, const SpecFork& fk) {
   static thread_local SpecParams<CAP> p;
   std::memset(&p, 0, sizeof(p));
   p.z = z; p.w = w; p.draft_tokens = dt;
@@ -729,12 +744,12 @@ int run_spec_cap(const SpecPlan& pl, int dtype, const void* z, const void* w, co
     p.topk_idx = sd.topk_idx;
     p.topk_q = sd.topk_q;
     p.topk = sd.topk;
-    return dtype == DIPSD_BF16 ? launch_spec_reg<__nv_bfloat16, CAP, true>(pl, p, s, pdl)
-                               : launch_spec_reg<float, CAP, true>(pl, p, s, pdl);
+    return dtype == DIPSD_BF16 ? launch_spec_reg<__nv_bfloat16, CAP, true>(pl, p, s, pdl, fk)
+                               : launch_spec_reg<float, CAP, true>(pl, p, s, pdl, fk);
   }
   if (pl.nk1)
-    return dtype == DIPSD_BF16 ? launch_spec_reg<__nv_bfloat16, CAP, false>(pl, p, s, pdl)
-                               : launch_spec_reg<float, CAP, false>(pl, p, s, pdl);
+    return dtype == DIPSD_BF16 ? launch_spec_reg<__nv_bfloat16, CAP, false>(pl, p, s, pdl, fk)
+                               : launch_spec_reg<float, CAP, false>(pl, p, s, pdl, fk);
   if (dtype == DIPSD_BF16)
     return pl.vec == 8 ? launch_spec_t<__nv_bfloat16, 8, CAP>(pl, p, s, pdl)
                        : launch_spec_t<__nv_bfloat16, 1, CAP>(pl, p, s, pdl);
@@ -743,12 +758,56 @@ int run_spec_cap(const SpecPlan& pl, int dtype, const void* z, const void* w, co
 
 int run_spec(const SpecPlan& pl, int dtype, const void* z, const void* w, const int* dt, uint64_t seed,
              const int* uid, int* acc, int* offs, int* toks, float* probs, unsigned* status, uint8_t* region,
-             cudaStream_t s, bool pdl, const SparseDraft& sd = SparseDraft{}) {
+             cudaStream_t s, bool pdl, const SparseDraft& sd = SparseDraft{}, const SpecFork& fk = SpecFork{}) {
   if (pl.B <= kCapSmall)
     return run_spec_cap<kCapSmall>(pl, dtype, z, w, dt, seed, uid, acc, offs, toks, probs, status, region, s, pdl,
-                                   sd);
+                                   sd, fk);
   return run_spec_cap<kCapLarge>(pl, dtype, z, w, dt, seed, uid, acc, offs, toks, probs, status, region, s, pdl,
-                                 sd);
+                                 sd, fk);
+}
+
+// The second stream and the two events verify_batch forks onto, one set per
+// host thread, device and caller stream (a few kept, made on first use).
+// Nothing is made while the caller's stream is being captured: such a call
+// runs on the one stream.  They live until the thread exits.
+struct ForkSet {
+  int dev = -1;
+  cudaStream_t caller = nullptr, aux = nullptr;
+  cudaEvent_t fork = nullptr, join = nullptr;
+};
+
+bool fork_set(cudaStream_t s, ForkSet** out) {
+  constexpr int kSets = 8;
+  static thread_local ForkSet sets[kSets];
+  static thread_local int next_slot = 0;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  for (ForkSet& f : sets)
+    if (f.aux && f.dev == dev && f.caller == s) {
+      *out = &f;
+      return true;
+    }
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(s, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone) return false;
+  ForkSet& f = sets[next_slot];
+  next_slot = (next_slot + 1) % kSets;
+  if (f.aux) {  // the oldest set goes to the new caller stream (queued work finishes first)
+    cudaStreamDestroy(f.aux);
+    cudaEventDestroy(f.fork);
+    cudaEventDestroy(f.join);
+    f = ForkSet{};
+  }
+  if (cudaStreamCreateWithFlags(&f.aux, cudaStreamNonBlocking) != cudaSuccess ||
+      cudaEventCreateWithFlags(&f.fork, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&f.join, cudaEventDisableTiming) != cudaSuccess) {
+    cudaGetLastError();
+    f = ForkSet{};
+    return false;
+  }
+  f.dev = dev;
+  f.caller = s;
+  *out = &f;
+  return true;
 }
 
 // Philox key word 1 of every user: a non-negative user id.
@@ -1124,18 +1183,28 @@ static int verify_batch_impl(int B, const int* h_members, int M, const int* h_L_
   uint8_t* ws = static_cast<uint8_t*>(d_workspace);
   unsigned* status = reinterpret_cast<unsigned*>(ws);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  // The two stages share no data.  spec_verify goes first; the attention
-  // grid launches as soon as the sampling kernel has passed its own wait
-  // (so everything before this call is complete), streams the KV cache
-  // while the sampling kernel's per-user descents finish, and waits for
-  // that kernel only before it exits.
-  // each member's Philox key word 1 is its index in the per-user tables
+  // The two stages share no data.  The statistics pass runs first, alone
+  // (it wants all of the HBM bandwidth); then the attention grid on the
+  // caller's stream and, beside it on a second stream, the decision and
+  // sampling kernels, latency-bound chains that need little bandwidth; the
+  // call's last operation joins the second stream back into the caller's.
+  // Without a second stream (a caller stream first seen inside a capture, the
+  // scalar path, or a test's choice) it is one stream: spec_verify, then the
+  // attention grid, which starts as soon as the sampling kernel has passed
+  // its own wait and waits for that kernel only before it exits.
+  // Each member's Philox key word 1 is its index in the per-user tables.
+  ForkSet* fs = nullptr;
+  const bool forked = sp.nk1 > 0 && plan_override(DIPSD_TEST_BATCH_FORK) != 2 && fork_set(s, &fs);
   st = run_spec(sp, logit_dtype, d_target_logits, d_draft_logits, d_draft_tokens, seed, h_members, d_accept_len,
-                d_out_offsets, d_out_tokens, d_draft_probs, status, ws + kHeaderBytes + attn_region, s, true);
+                d_out_offsets, d_out_tokens, d_draft_probs, status, ws + kHeaderBytes + attn_region, s, true,
+                SparseDraft{}, forked ? SpecFork{fs->aux, fs->fork} : SpecFork{});
   if (st != DIPSD_OK) return st;
   st = run_attention(ap, d_q, d_k_cache, d_v_cache, num_blocks, d_block_table_all, max_blocks, softmax_scale,
-                     d_attn_out, status, ws + kHeaderBytes, s, true, app, true);
-  return st != DIPSD_OK ? st : cuda_status();
+                     d_attn_out, status, ws + kHeaderBytes, s, !forked, app, !forked);
+  if (st != DIPSD_OK) return st;
+  if (forked && (cudaEventRecord(fs->join, fs->aux) != cudaSuccess || cudaStreamWaitEvent(s, fs->join, 0) != cudaSuccess))
+    return DIPSD_ERR_CUDA;
+  return cuda_status();
 }
 
 int dipsd_verify_batch(int B, const int* h_members, int M, const int* h_L_all, const int* h_ctx_all,

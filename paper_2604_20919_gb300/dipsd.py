@@ -41,7 +41,7 @@ EXPORTS = (
 NOALLOC_MAX_POSITIONS = 4096
 # dipsd_test_set_override codes
 TEST_OVERRIDES = {"attn_split_tiles": 1, "attn_cluster": 2, "attn_persist": 3, "attn_grid": 4,
-                  "spec_nk1": 5, "spec_nk2": 6, "spec_grid1": 7}
+                  "spec_nk1": 5, "spec_nk2": 6, "spec_grid1": 7, "batch_fork": 8}
 
 _lib: Optional[ctypes.CDLL] = None
 _i32p = ctypes.c_void_p  # host int32 arrays, passed by address

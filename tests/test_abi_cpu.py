@@ -136,7 +136,7 @@ def test_test_overrides_are_explicit(lib):
         assert dipsd.dipsd_verify_attention_plan(L, ctx, 64, 8, 128, 152)["cluster"] == 3
     assert dipsd.dipsd_verify_attention_plan(L, ctx, 64, 8, 128, 152)["cluster"] == base["cluster"]
     assert lib.dipsd_test_set_override(0, 1) == 1
-    assert lib.dipsd_test_set_override(8, 1) == 1
+    assert lib.dipsd_test_set_override(9, 1) == 1
     assert lib.dipsd_test_set_override(1, -1) == 1
 
 

@@ -40,14 +40,18 @@ def test_pipelined_stages_on_two_streams(cuda_lib):
         print(f"stage {n}: {st}, attention max err {err:.3e}")
 
 
-def test_batch_matches_separate_calls(cuda_lib):
+@pytest.mark.parametrize("fork", [1, 2])
+def test_batch_matches_separate_calls(cuda_lib, fork):
+    """verify_batch equals the two separate calls, with the decision and
+    sampling kernels on the library's second stream (1) or on the caller's (2)."""
     b = make_config(2, seed=4)
     g = lambda t: t.to(DEV)
     q, kc, vc, bt = g(b.q), g(b.k_cache), g(b.v_cache), g(b.block_table)
     z, w, d = g(b.target_logits), g(b.draft_logits), g(b.draft_tokens)
     attn_a = cuda_lib.dipsd_verify_attention(b.L, b.ctx, q, kc, vc, bt, b.scale)
     sv = cuda_lib.dipsd_spec_verify(b.L, b.members, b.seed, z, w, d)
-    res = cuda_lib.dipsd_verify_batch(b.members, b.L, b.ctx, q, kc, vc, bt, b.scale, z, w, d, b.seed)
+    with cuda_lib.plan_override(batch_fork=fork):
+        res = cuda_lib.dipsd_verify_batch(b.members, b.L, b.ctx, q, kc, vc, bt, b.scale, z, w, d, b.seed)
     torch.cuda.synchronize()
     assert torch.equal(attn_a, res[0])
     for x, y in zip(valid_spec_outputs(*sv), valid_spec_outputs(*res[1:])):
@@ -78,3 +82,36 @@ def test_batch_with_permuted_membership(cuda_lib):
                                       np.abs(b.v_cache.double().numpy()), b.block_table.numpy(), b.ctx, b.L, b.scale)
     check_attention(attn, ref, ref_abs)
     check_spec(b, acc, offs, toks, probs)
+
+
+def test_batch_captured_in_a_graph(cuda_lib):
+    """verify_batch captured into a CUDA graph (both streams) and replayed:
+    the replays give the outputs of a plain call."""
+    b = make_config(2, seed=9)
+    g = lambda t: t.to(DEV)
+    q, kc, vc, bt = g(b.q), g(b.k_cache), g(b.v_cache), g(b.block_table)
+    z, w, d = g(b.target_logits), g(b.draft_logits), g(b.draft_tokens)
+    ws = cuda_lib.workspace(cuda_lib.dipsd_verify_batch_workspace_size(b.members, b.L, b.ctx, b.Hq, b.Hkv, b.D, b.V),
+                            DEV)
+    attn = torch.empty_like(q)
+    outs = cuda_lib.spec_outputs(b.L, DEV)
+    call = lambda: cuda_lib.dipsd_verify_batch(b.members, b.L, b.ctx, q, kc, vc, bt, b.scale, z, w, d, b.seed,
+                                               attn_out=attn, outputs=outs, ws=ws)
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        call()  # the first call from this stream, outside the capture
+    torch.cuda.synchronize()
+    ref = [attn.clone()] + [t.clone() for t in valid_spec_outputs(*outs)]
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=s):  # a stream that made a plain call first
+        call()
+    for _ in range(3):
+        attn.zero_()
+        for t in outs[:3]:
+            t.fill_(-1)
+        graph.replay()
+        torch.cuda.synchronize()
+        got = [attn] + valid_spec_outputs(*outs)
+        for x, y in zip(ref, got):
+            assert torch.equal(x, y)
+    assert cuda_lib.device_status(ws) == 0
