@@ -1184,10 +1184,11 @@ static int verify_batch_impl(int B, const int* h_members, int M, const int* h_L_
   unsigned* status = reinterpret_cast<unsigned*>(ws);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   // The two stages share no data.  The statistics pass runs first, alone
-  // (it wants all of the HBM bandwidth); then the attention grid on the
-  // caller's stream and, beside it on a second stream, the decision and
-  // sampling kernels, latency-bound chains that need little bandwidth; the
-  // call's last operation joins the second stream back into the caller's.
+  // (it wants all of the HBM bandwidth: an attention grid started while it
+  // drains measured slower); then the attention grid on the caller's stream
+  // and, beside it on a second stream, the decision and sampling kernels,
+  // latency-bound chains that need little bandwidth; the call's last
+  // operation joins the second stream back into the caller's.
   // Without a second stream (a caller stream first seen inside a capture, the
   // scalar path, or a test's choice) it is one stream: spec_verify, then the
   // attention grid, which starts as soon as the sampling kernel has passed

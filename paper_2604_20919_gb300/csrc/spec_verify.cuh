@@ -670,8 +670,12 @@ spec_stats_kernel(const __grid_constant__ SpecParams<CAP> p) {
   const int W = gridDim.x * kRegWarps;
   int item = blockIdx.x * kRegWarps + (threadIdx.x >> 5);
   pdl_wait_prior_grid();
-  pdl_launch_dependents();
-  if (item >= p.n_items1) return;
+  // (the dependent grid is released as each CTA finishes its segments: the
+  // decision kernel's CTAs then take no SM slot while this pass streams)
+  if (item >= p.n_items1) {
+    pdl_launch_dependents();
+    return;
+  }
   constexpr int KG = NK < 4 ? NK : 4;
   StatSeg<T> g = stat_seg<T, NK, CAP, SP>(p, item, lane);
   uint4 r[NK];
@@ -702,6 +706,7 @@ spec_stats_kernel(const __grid_constant__ SpecParams<CAP> p) {
     g = ng;
     xd = nxd;
   }
+  pdl_launch_dependents();
 }
 
 // One warp per verify position: the row sums from the statistics pass's
