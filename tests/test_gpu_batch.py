@@ -115,3 +115,28 @@ def test_batch_captured_in_a_graph(cuda_lib):
         for x, y in zip(ref, got):
             assert torch.equal(x, y)
     assert cuda_lib.device_status(ws) == 0
+
+
+def test_batch_from_many_streams(cuda_lib):
+    """Calls from more caller streams than the library keeps second streams
+    for (each new stream takes over the oldest set): every call still gives
+    the outputs of the first, and the status word stays clear."""
+    b = make_config(2, seed=11)
+    g = lambda t: t.to(DEV)
+    q, kc, vc, bt = g(b.q), g(b.k_cache), g(b.v_cache), g(b.block_table)
+    z, w, d = g(b.target_logits), g(b.draft_logits), g(b.draft_tokens)
+    ref = cuda_lib.dipsd_verify_batch(b.members, b.L, b.ctx, q, kc, vc, bt, b.scale, z, w, d, b.seed)
+    torch.cuda.synchronize()
+    ref = [ref[0]] + valid_spec_outputs(*ref[1:])
+    streams = [torch.cuda.Stream() for _ in range(10)]
+    results = []
+    for _ in range(2):
+        for s in streams:
+            with torch.cuda.stream(s):
+                results.append(cuda_lib.dipsd_verify_batch(b.members, b.L, b.ctx, q, kc, vc, bt, b.scale, z, w,
+                                                           d, b.seed, stream=s))
+    torch.cuda.synchronize()
+    for res in results:
+        got = [res[0]] + valid_spec_outputs(*res[1:])
+        for x, y in zip(ref, got):
+            assert torch.equal(x, y)
