@@ -155,8 +155,9 @@ typedef struct {
   int grid;        /* CTAs launched: n_items, or (chunk_pages > 0) the chunks */
   int cluster;     /* > 1: every user's KV in `cluster` splits that merge
                       inside one thread-block cluster; 0 otherwise */
-  int n_merge;     /* (verify token, query head) rows the separate merge
-                      kernel visits after the grid (0: no merge launch) */
+  int n_merge;     /* (verify token, query head) rows whose KV stream has
+                      more than one split, combined by a merge kernel after
+                      the grid (0: no merge launch) */
   int stream_chunks; /* > 0: the persistent grid's chunks (CTAs) */
   size_t ws_bytes; /* workspace bytes of this plan past the status header */
 } dipsd_attention_plan;

@@ -40,6 +40,17 @@ struct AttnUser {
   int n_rb;       // row blocks
 };
 
+// A page stream cut by chunk bounds (persistent grid), as its merge reads
+// it: written by the CTA that runs the stream's first split, read by the
+// merge kernel after the grid.  Partial row of split s and row r of the
+// stream's row block: part_row0 + s * step + r; output row of row rg =
+// row0 + r (t = rg / G, g = rg % G): out_base + t * Hq + g.
+struct MergeDesc {
+  long long part_row0;
+  long long out_base;
+  int step, nsplit, nrows, row0;
+};
+
 template <int CAP>
 struct AttnParams {
   const __nv_bfloat16* q;
@@ -69,6 +80,16 @@ struct AttnParams {
   int item_off[CAP + 1];
   int page_off[CAP + 1];  // page streams: first page of user i's streams
   int chunk_bound[kMaxChunks + 1];  // page streams: chunk b is [chunk_bound[b], chunk_bound[b + 1])
+  // page streams, per chunk b: the user of its first page, how many chunks
+  // back the stream of its first page starts, and how many chunks ahead the
+  // stream of its last page ends (so no CTA searches the chunk bounds)
+  short chunk_user[kMaxChunks];
+  unsigned char chunk_c0_back[kMaxChunks];
+  unsigned char chunk_c1_fwd[kMaxChunks];
+  // page streams: per chunk, the index of the cut stream that starts in it
+  // (255: none); its merge descriptor goes to merge_desc[index]
+  unsigned char chunk_cut[kMaxChunks];
+  MergeDesc* merge_desc;
   int merge_off[CAP + 1];
   long long part_off[CAP];  // first partial row of the user (multi-split users)
   AttnUser u[CAP];
@@ -111,49 +132,52 @@ __device__ __forceinline__ Work work_of_item(const AttnParams<CAP>& p, int item)
   return w;
 }
 
-// The chunk that holds page `pos` (page streams).
+// Page-stream decoding.  Streams of user i: index sidx = rb * Hkv + h, each
+// pages_of(U) pages, from page page_off[i].  The piece of stream (ui, sidx)
+// that starts at page `pos` in chunk `cta` (which ends at page `hi`), the
+// stream starting in chunk c0: its splits run from chunk c0 to the chunk
+// where it ends, which is `cta` unless the stream runs past `hi` (then this
+// is the chunk's last piece, and the host recorded that chunk).
 template <int CAP>
-__device__ __forceinline__ int chunk_of(const AttnParams<CAP>& p, int pos) {
-  int lo = 0, hi = p.n_chunks - 1;  // last b with chunk_bound[b] <= pos
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (p.chunk_bound[mid] <= pos) lo = mid; else hi = mid - 1;
-  }
-  return lo;
-}
-
-// Splits of the page stream that starts at page s0 and holds np pages: the
-// chunks it touches, the first of them c0.
-template <int CAP>
-__device__ __forceinline__ int stream_splits(const AttnParams<CAP>& p, int s0, int np, int* c0) {
-  *c0 = chunk_of<CAP>(p, s0);
-  return chunk_of<CAP>(p, s0 + np - 1) - *c0 + 1;
-}
-
-// Page-stream decoding: the piece that starts at page `pos` of CTA `cta`,
-// whose chunk ends at page `hi`.  Streams of user i: index (rb * Hkv + h),
-// each pages_of(U) pages.
-template <int CAP>
-__device__ __forceinline__ Work work_of_page(const AttnParams<CAP>& p, int pos, int cta, int hi) {
+__device__ __forceinline__ Work piece_of_stream(const AttnParams<CAP>& p, int ui, int sidx, int pos, int c0,
+                                                int cta, int hi) {
   Work w;
-  w.ui = find_user<CAP>(p.page_off, p.B, pos);
-  const AttnUser& U = p.u[w.ui];
+  const AttnUser& U = p.u[ui];
   const int np = pages_of(U);
-  const int sidx = (pos - p.page_off[w.ui]) / np;
+  const int s0 = p.page_off[ui] + sidx * np;
+  w.ui = ui;
   w.h = sidx % p.Hkv;
   w.rb = sidx / p.Hkv;
-  const int s0 = p.page_off[w.ui] + sidx * np;
   w.next = min(hi, s0 + np);
   w.kv_begin = (pos - s0) * kPage;
   w.kv_end = min((w.next - s0) * kPage, U.kv_len);
-  int c0;
-  w.nsplit = stream_splits<CAP>(p, s0, np, &c0);
+  const int c1 = s0 + np <= hi ? cta : cta + p.chunk_c1_fwd[cta];
+  w.nsplit = c1 - c0 + 1;
   w.split = cta - c0;
   return w;
 }
+// The first piece of chunk `cta`: it starts at the chunk's first page.
+template <int CAP>
+__device__ __forceinline__ Work first_piece(const AttnParams<CAP>& p, int cta, int hi) {
+  const int pos = p.chunk_bound[cta];
+  const int ui = p.chunk_user[cta];
+  const int sidx = (pos - p.page_off[ui]) / pages_of(p.u[ui]);
+  return piece_of_stream<CAP>(p, ui, sidx, pos, cta - p.chunk_c0_back[cta], cta, hi);
+}
+// The piece after w in chunk `cta` (w.next < hi): the next stream, from its
+// first page, in this chunk.
+template <int CAP>
+__device__ __forceinline__ Work next_piece(const AttnParams<CAP>& p, const Work& w, int cta, int hi) {
+  int ui = w.ui, sidx = w.rb * p.Hkv + w.h + 1;
+  if (sidx == p.u[ui].n_rb * p.Hkv) {
+    ++ui;
+    sidx = 0;
+  }
+  return piece_of_stream<CAP>(p, ui, sidx, w.next, cta, cta, hi);
+}
 
 // Combines the KV splits of every (verify token, query head) row of users
-// with more than one split: m = max_s m_s, w_s = 2^(m_s - m),
+// with more than one split (one CTA per item plans): m = max_s m_s, w_s = 2^(m_s - m),
 // out = sum_s w_s o_s / sum_s w_s l_s.  One warp per row: lane k holds the
 // (m, l) of splits k, k + 32, ..., the weights reach every lane by shuffle,
 // and the O rows of eight splits are loaded before any is used.
@@ -171,13 +195,7 @@ verify_attention_merge_kernel(const __grid_constant__ AttnParams<CAP> p) {
   const int t = local / p.Hq, hq = local % p.Hq;
   const int h = hq / p.G, g = hq % p.G;
   const int M = p.G * U.T;
-  int ns = U.nsplit;
-  if (p.n_chunks > 0) {  // page streams: this row's stream may be whole
-    const int np = pages_of(U), sidx = ((t * p.G + g) / 128) * p.Hkv + h;
-    int c0;
-    ns = stream_splits<CAP>(p, p.page_off[ui] + sidx * np, np, &c0);
-    if (ns == 1) return;  // written by its CTA
-  }
+  const int ns = U.nsplit;
   // partial row of split s: base + s * stride
   const long long base = p.part_off[ui] + static_cast<long long>(h) * M + t * p.G + g;
   const long long stride = static_cast<long long>(p.Hkv) * M;
@@ -232,6 +250,80 @@ verify_attention_merge_kernel(const __grid_constant__ AttnParams<CAP> p) {
 #pragma unroll
   for (int k = 0; k < kPer; k += 2)
     *reinterpret_cast<uint32_t*>(out + k) = pack_bf16x2(acc[k] * inv, acc[k + 1] * inv);
+}
+
+// Combines the splits of the cut page streams of a persistent grid (the
+// same formula as above, as a running merge: the weights are rescaled when a
+// later split raises the maximum): CTA (k, c) takes cut stream k and its
+// 32-column slice c, one thread per row of the stream's row block.  A round
+// of loads brings the (m, l) and the O slices of two splits, so a stream cut
+// once costs the descriptor load and one round.
+template <int D, int CAP>
+__global__ void __launch_bounds__(128)
+verify_attention_merge_streams_kernel(const __grid_constant__ AttnParams<CAP> p) {
+  pdl_wait_prior_grid();
+  pdl_launch_dependents();
+  const MergeDesc* dp = p.merge_desc + blockIdx.x;
+  const int nrows = __ldcg(&dp->nrows);
+  const int r = static_cast<int>(threadIdx.x);
+  if (r >= nrows) return;
+  const long long row = __ldcg(&dp->part_row0) + r;
+  const long long step = __ldcg(&dp->step);
+  const int ns = __ldcg(&dp->nsplit);
+  const int col = blockIdx.y * 32;
+  float m = -INFINITY, l = 0.f;
+  float acc[32];
+#pragma unroll
+  for (int k = 0; k < 32; ++k) acc[k] = 0.f;
+  for (int s0 = 0; s0 < ns; s0 += 2) {
+    float2 ml[2];
+    float4 v[2][8];
+#pragma unroll
+    for (int b = 0; b < 2; ++b) {
+      ml[b] = make_float2(-INFINITY, 0.f);
+      if (s0 + b < ns) {
+        const long long rs = row + (s0 + b) * step;
+        ml[b] = __ldcg(p.part_ml + rs);
+        const float4* po = reinterpret_cast<const float4*>(p.part_o + rs * D + col);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) v[b][k] = __ldcg(po + k);
+      }
+    }
+    // an empty split (no visible key: m = -inf, l = 0) weighs nothing
+    const bool ok0 = ml[0].x > -INFINITY && ml[0].y > 0.f, ok1 = ml[1].x > -INFINITY && ml[1].y > 0.f;
+    const float mn = fmaxf(m, fmaxf(ok0 ? ml[0].x : -INFINITY, ok1 ? ml[1].x : -INFINITY));
+    if (mn > m) {
+      const float f = m == -INFINITY ? 0.f : fast_exp2(m - mn);
+#pragma unroll
+      for (int k = 0; k < 32; ++k) acc[k] *= f;
+      l *= f;
+      m = mn;
+    }
+#pragma unroll
+    for (int b = 0; b < 2; ++b) {
+      if (b == 0 ? ok0 : ok1) {
+        const float w = fast_exp2(ml[b].x - m);
+        l += w * ml[b].y;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          acc[4 * k] += w * v[b][k].x;
+          acc[4 * k + 1] += w * v[b][k].y;
+          acc[4 * k + 2] += w * v[b][k].z;
+          acc[4 * k + 3] += w * v[b][k].w;
+        }
+      }
+    }
+  }
+  const float inv = l > 0.f ? 1.f / l : 0.f;
+  const int rg = __ldcg(&dp->row0) + r;
+  const int t = rg / p.G, g = rg % p.G;
+  uint4* dst = reinterpret_cast<uint4*>(p.out + (__ldcg(&dp->out_base) + static_cast<long long>(t) * p.Hq + g) * D + col);
+#pragma unroll
+  for (int k = 0; k < 4; ++k)
+    dst[k] = make_uint4(pack_bf16x2(acc[8 * k] * inv, acc[8 * k + 1] * inv),
+                        pack_bf16x2(acc[8 * k + 2] * inv, acc[8 * k + 3] * inv),
+                        pack_bf16x2(acc[8 * k + 4] * inv, acc[8 * k + 5] * inv),
+                        pack_bf16x2(acc[8 * k + 6] * inv, acc[8 * k + 7] * inv));
 }
 
 }  // namespace dipsd

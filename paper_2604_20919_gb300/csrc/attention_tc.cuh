@@ -129,13 +129,13 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
   // phases run on across them (global tile index g0 + j).
   const int chunk_lo = PERSIST ? p.chunk_bound[blockIdx.x] : static_cast<int>(blockIdx.x);
   const int chunk_hi = PERSIST ? p.chunk_bound[blockIdx.x + 1] : 0;
-  auto decode = [&](int w) {
-    return PERSIST ? work_of_page<CAP>(p, w, blockIdx.x, chunk_hi) : work_of_item<CAP>(p, w);
-  };
+  // (pieces after a CTA's first follow from the one before: the next stream)
   int ui, split, nsplit, h, rb, M, row0, kv_begin, kv_end, ntiles, split_pages_n, next_w;
   AttnUser U;
-  auto set_item = [&](int w) {
-    const Work W = decode(w);
+  Work unit = PERSIST ? first_piece<CAP>(p, blockIdx.x, chunk_hi) : work_of_item<CAP>(p, blockIdx.x);
+  auto following = [&]() { return next_piece<CAP>(p, unit, blockIdx.x, chunk_hi); };
+  auto set_item = [&](const Work& W) {
+    unit = W;
     ui = W.ui;
     U = p.u[ui];
     split = W.split;
@@ -155,7 +155,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
   };
   // is there work after the current unit (the loop tests it before set_item)
   auto more = [&]() { return PERSIST && next_w < chunk_hi; };
-  set_item(chunk_lo);
+  set_item(unit);
   auto tile_pages = [&](int j) { return min(kTcTile / kPage, split_pages_n - j * (kTcTile / kPage)); };
   // tile j holds new (appended) rows: keys [max(key0, C_i), min(key0 + 128, kv_end)).
   // The patch barriers are single-use: a launch that appends runs one item per CTA.
@@ -229,7 +229,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
     };
     int ahead = 0;  // the next unit's first page group, loaded one unit early
     for (int n = 0; alive && (n == 0 || more()); ++n) {
-      if (n > 0) set_item(next_w);
+      if (n > 0) set_item(following());
       const int g0 = issued;
       const int* bt = p.block_table + static_cast<size_t>(U.bt_row) * p.max_blocks;
       auto fetch = [&](int group) { return fetch_of(U.bt_row, kv_begin, kv_end, group); };
@@ -238,8 +238,18 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
       if (more()) {
         // the next unit's first page group, so its first loads do not wait
         // on a dependent block-table read at the boundary
-        const Work Wn = decode(next_w);
+        const Work Wn = following();
         ahead = fetch_of(p.u[Wn.ui].bt_row, Wn.kv_begin, Wn.kv_end, 0);
+        // and the Q rows of the next two units into L2: the softmax warps
+        // read a unit's Q one unit ahead, and a read that went to DRAM would
+        // queue behind this SM's K/V stream (~4 us) while they wait on it
+        auto prefetch_q = [&](const Work& W) {
+          const AttnUser& Un = p.u[W.ui];
+          if (lane < Un.T)
+            bulk_prefetch_l2(p.q + (static_cast<size_t>(Un.q_off + lane) * p.Hq + W.h * p.G) * D, p.G * D * 2);
+        };
+        prefetch_q(Wn);
+        if (Wn.next < chunk_hi) prefetch_q(next_piece<CAP>(p, Wn, blockIdx.x, chunk_hi));
       }
       for (int j = 0; j < ntiles; ++j) {
         const int gj = g0 + j;
@@ -349,7 +359,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
       bool ok = true;
       int g0 = 0;  // global index of the item's first tile
       for (int n = 0; ok && (n == 0 || more()); ++n) {
-        if (n > 0) set_item(next_w);
+        if (n > 0) set_item(following());
         // Q of this unit is in TMEM buffer n & 1 (written one unit ahead)
         ok = mbar_wait(&q_ready[n & 1], (n >> 1) & 1, p.status);
         const uint32_t tQn = tQ + (n & 1) * kQCols;
@@ -425,8 +435,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
     int g0 = 0;  // global index of the item's first tile
     // Q row of the unit starting at w -> TMEM buffer qb, lane r, as bf16
     // pairs (column c holds elements 2c, 2c+1); padding rows are zero
-    auto write_q = [&](int w, int qb) {
-      const Work Wj = decode(w);
+    auto write_q = [&](const Work& Wj, int qb) {
       const AttnUser Uj = p.u[Wj.ui];
       const int hj = Wj.h, rgj = Wj.rb * 128 + r;
       const bool validj = rgj < p.G * Uj.T;
@@ -452,7 +461,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
       if (lane == 0) mbar_arrive(&q_ready[qb]);
     };
     for (int n = 0; ok && (n == 0 || more()); ++n) {
-      if (n > 0) set_item(next_w);
+      if (n > 0) set_item(following());
       const int rg = row0 + r;  // row within the user
       const bool valid = rg < M;
       const int t = rg / p.G, g = rg % p.G;
@@ -463,9 +472,9 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
       // (off the path from this item's start to its first P V); the buffer's
       // previous user, item n - 1, has its products done: its o_final was
       // waited for.
-      if (n == 0) write_q(chunk_lo, 0);
+      if (n == 0) write_q(unit, 0);
       const bool prefetch = more();
-      const int w_next = next_w;
+      const Work w_next = prefetch ? following() : unit;
       if (prefetch && ntiles == 0) write_q(w_next, (n + 1) & 1);
 
       const int last_vis = min(U.ctx + t, kv_end - 1);  // last key of this row in this split
@@ -606,6 +615,19 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
           }
         }
         if (valid && nsplit > 1) p.part_ml[prow_idx] = make_float2(m, l);
+      }
+      if constexpr (PERSIST) {
+        // the first split of a cut stream leaves the stream's merge descriptor
+        if (nsplit > 1 && split == 0 && threadIdx.x == 64) {
+          MergeDesc dsc;
+          dsc.part_row0 = p.part_off[ui] + static_cast<long long>(h) * M + row0;
+          dsc.out_base = static_cast<long long>(U.q_off) * p.Hq + h * p.G;
+          dsc.step = p.Hkv * M;
+          dsc.nsplit = nsplit;
+          dsc.nrows = min(128, M - row0);
+          dsc.row0 = row0;
+          p.merge_desc[p.chunk_cut[blockIdx.x]] = dsc;
+        }
       }
       tc_fence_before();
       g0 += ntiles;

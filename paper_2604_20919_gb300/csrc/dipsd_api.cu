@@ -28,6 +28,9 @@ constexpr size_t kCounterBytes = (kCounterWords * sizeof(unsigned) + 255) / 256 
 constexpr size_t kHeaderBytes = kStatusBytes + kCounterBytes;
 constexpr int kCapSmall = 64;
 constexpr int kCapLarge = kMaxUsers;
+// kernel parameters are limited to 32764 bytes (the attention grid also
+// takes its two tensor maps)
+static_assert(sizeof(AttnParams<kCapLarge>) + 2 * sizeof(CUtensorMap) <= 32764, "attention parameters");
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
@@ -149,6 +152,14 @@ struct AttnPlan {
   int n_items = 0, n_merge = 0;
   int n_chunks = 0, total_pages = 0;  // page streams (persistent grid): chunks, all pages
   std::vector<int> chunk_bound;        // chunk b: pages [chunk_bound[b], chunk_bound[b + 1])
+  // per chunk: the user of its first page; chunks back to where the stream of
+  // its first page starts; chunks ahead to where the stream of its last ends
+  std::vector<short> chunk_user;
+  std::vector<unsigned char> chunk_c0_back, chunk_c1_fwd;
+  // page streams cut by chunk bounds (merged after the grid): per chunk the
+  // index of the cut stream that starts in it (255: none), and their count
+  std::vector<unsigned char> chunk_cut;
+  int n_cut = 0;
   int grid = 0;     // CTAs launched: n_items, or fewer that each walk several items
   int cluster = 0;  // > 1: splits merged inside a thread-block cluster of this size
   long long part_rows = 0;
@@ -406,11 +417,51 @@ void plan_attention(int B, const int* L, const int* ctx, const int* bt_rows, int
   pl.item_off[B] = static_cast<int>(items);
   pl.merge_off[B] = static_cast<int>(merge);
   pl.page_off[B] = static_cast<int>(pos_pages);
+  long long merge_rows = 0;
+  if (persist) {
+    // where the streams at each chunk's two ends start and end (the kernel
+    // walks a chunk's later pieces stream by stream, with no search)
+    const int nc = pl.n_chunks;
+    auto chunk_at = [&](int pos) {
+      return static_cast<int>(std::upper_bound(sk_bound.begin(), sk_bound.end() - 1, pos) - sk_bound.begin()) - 1;
+    };
+    auto stream_at = [&](int pos, int* ui, int* s0, int* np) {  // the stream holding page pos
+      *ui = static_cast<int>(std::upper_bound(pl.page_off.begin(), pl.page_off.begin() + B, pos) -
+                             pl.page_off.begin()) - 1;
+      *np = (pl.u[*ui].kv_len + kPage - 1) / kPage;
+      const int k = std::min((pos - pl.page_off[*ui]) / *np, pl.u[*ui].n_rb * Hkv - 1);
+      *s0 = pl.page_off[*ui] + k * *np;
+    };
+    pl.chunk_user.assign(nc, 0);
+    pl.chunk_c0_back.assign(nc, 0);
+    pl.chunk_c1_fwd.assign(nc, 0);
+    pl.chunk_cut.assign(nc, 255);
+    for (int b = 0; b < nc; ++b) {
+      const int lo = sk_bound[b], hi = sk_bound[b + 1];
+      if (lo >= hi) continue;  // an empty chunk runs no piece
+      int ui, s0, np;
+      stream_at(lo, &ui, &s0, &np);
+      pl.chunk_user[b] = static_cast<short>(ui);
+      pl.chunk_c0_back[b] = static_cast<unsigned char>(b - chunk_at(s0));
+      stream_at(hi - 1, &ui, &s0, &np);
+      const int c1 = chunk_at(s0 + np - 1);
+      pl.chunk_c1_fwd[b] = static_cast<unsigned char>(c1 - b);
+      if (c1 > b && chunk_at(s0) == b) {  // a stream that starts here and runs on: cut
+        const int sidx = (s0 - pl.page_off[ui]) / np;
+        pl.chunk_cut[b] = static_cast<unsigned char>(pl.n_cut++);
+        merge_rows += std::min(rows_cta, pl.G * pl.u[ui].T - (sidx / Hkv) * rows_cta);
+      }
+    }
+  }
   pl.n_items = static_cast<int>(items);
   pl.grid = persist ? sk_grid : pl.n_items;
-  pl.n_merge = static_cast<int>(merge);
+  // rows whose stream has more than one split: every row of a split user
+  // (one CTA per item), the rows of the cut streams (page streams)
+  pl.n_merge = static_cast<int>(persist ? merge_rows : merge);
   pl.part_rows = part;
-  pl.ws_bytes = part ? align_up(part * sizeof(float2), 256) + align_up(part * D * sizeof(float), 256) : 0;
+  pl.ws_bytes = part ? align_up(part * sizeof(float2), 256) + align_up(part * D * sizeof(float), 256) +
+                           align_up(pl.n_cut * sizeof(MergeDesc), 256)
+                     : 0;
 }
 
 // KV-append inputs of one call (all null: the cache already holds the rows).
@@ -428,13 +479,22 @@ void fill_attn_params(AttnParams<CAP>& p, const AttnPlan& pl, const void* q, voi
   p.block_table = bt;
   p.part_ml = reinterpret_cast<float2*>(region);
   p.part_o = reinterpret_cast<float*>(region + align_up(pl.part_rows * sizeof(float2), 256));
+  p.merge_desc = reinterpret_cast<MergeDesc*>(region + align_up(pl.part_rows * sizeof(float2), 256) +
+                                              align_up(pl.part_rows * pl.D * sizeof(float), 256));
   p.status = status;
   p.cluster = pl.cluster;
   p.B = pl.B; p.Hq = pl.Hq; p.Hkv = pl.Hkv; p.G = pl.G; p.max_blocks = max_blocks;
   p.n_items = pl.n_items; p.n_merge = pl.n_merge;
   p.n_chunks = pl.n_chunks; p.total_pages = pl.total_pages;
-  if (pl.n_chunks > 0)
+  if (pl.n_chunks > 0) {
     for (int b = 0; b <= pl.n_chunks; ++b) p.chunk_bound[b] = pl.chunk_bound[b];
+    for (int b = 0; b < pl.n_chunks; ++b) {
+      p.chunk_user[b] = pl.chunk_user[b];
+      p.chunk_c0_back[b] = pl.chunk_c0_back[b];
+      p.chunk_c1_fwd[b] = pl.chunk_c1_fwd[b];
+    }
+    for (int b = 0; b < pl.n_chunks; ++b) p.chunk_cut[b] = pl.chunk_cut[b];
+  }
   p.scale_log2 = scale * 1.4426950408889634f;
   for (int i = 0; i <= pl.B; ++i) {
     p.item_off[i] = pl.item_off[i];
@@ -459,9 +519,11 @@ int launch_attention_tc_t(const AttnPlan& pl, const AttnParams<CAP>& p, const CU
              p, tk, tv) != cudaSuccess)
     return DIPSD_ERR_CUDA;
   if (pl.n_merge > 0) {
-    auto mk = verify_attention_merge_kernel<D, CAP>;
-    if (launch(mk, dim3((pl.n_merge + 3) / 4), dim3(128), 0, s, 0, true, p) != cudaSuccess)
-      return DIPSD_ERR_CUDA;
+    const cudaError_t e =
+        persist ? launch(verify_attention_merge_streams_kernel<D, CAP>, dim3(static_cast<unsigned>(pl.n_cut), D / 32),
+                         dim3(128), 0, s, 0, true, p)
+                : launch(verify_attention_merge_kernel<D, CAP>, dim3((pl.n_merge + 3) / 4), dim3(128), 0, s, 0, true, p);
+    if (e != cudaSuccess) return DIPSD_ERR_CUDA;
   }
   return DIPSD_OK;
 }

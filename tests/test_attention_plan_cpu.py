@@ -22,11 +22,13 @@ def dipsd():
 
 
 def _page_streams(L, ctx, G, Hkv):
-    """(user, pages) of every (user, row block, KV head) stream, in the order
-    the persistent grid lays them back to back."""
+    """(user, pages, rows) of every (user, row block, KV head) stream, in the
+    order the persistent grid lays them back to back."""
     pages = -(-(np.asarray(ctx) + np.asarray(L) + 1) // PAGE)
-    rb = -(-(G * (np.asarray(L) + 1)) // ROWS_PER_ITEM)
-    return [(i, int(pages[i])) for i in range(len(L)) for _ in range(int(rb[i]) * Hkv)]
+    M = G * (np.asarray(L) + 1)
+    rb = -(-M // ROWS_PER_ITEM)
+    return [(i, int(pages[i]), int(min(ROWS_PER_ITEM, M[i] - r * ROWS_PER_ITEM)))
+            for i in range(len(L)) for r in range(int(rb[i])) for _ in range(Hkv)]
 
 
 def _check_plan(p, L, ctx, Hq, Hkv, D, num_sms, append, forced_cluster=False):
@@ -43,19 +45,22 @@ def _check_plan(p, L, ctx, Hq, Hkv, D, num_sms, append, forced_cluster=False):
         assert not append and not p["cluster"]
         bound = np.asarray(p["chunk_bound"])
         streams = _page_streams(L, ctx, G, Hkv)
-        total = sum(n for _, n in streams)
+        total = sum(n for _, n, _ in streams)
         assert p["grid"] == p["stream_chunks"] == len(bound) - 1 <= min(num_sms, 256)
         assert bound[0] == 0 and bound[-1] == total and (np.diff(bound) > 0).all()
         chunk_of = lambda pos: int(np.searchsorted(bound, pos, side="right")) - 1
-        pieces, ns_user, pos = 0, np.ones(len(L), dtype=int), 0
-        for i, n in streams:
+        pieces, ns_user, pos, cut_rows = 0, np.ones(len(L), dtype=int), 0, 0
+        for i, n, rows in streams:
             c = chunk_of(pos + n - 1) - chunk_of(pos) + 1
             pieces += c
             ns_user[i] = max(ns_user[i], c)
+            cut_rows += rows if c > 1 else 0
             pos += n
         assert p["n_items"] == pieces
         np.testing.assert_array_equal(ns, ns_user)
         split_users = ns_user > 1
+        # the merge visits the rows of the streams cut by a chunk bound
+        assert p["n_merge"] == cut_rows
     else:
         # every key of a user lies in exactly one split; only cluster plans may
         # carry trailing empty splits (every user then has exactly `cluster`)
@@ -72,10 +77,11 @@ def _check_plan(p, L, ctx, Hq, Hkv, D, num_sms, append, forced_cluster=False):
         assert p["n_items"] == int((ns * row_blocks * Hkv).sum())
         assert p["grid"] == p["n_items"]  # one CTA per item
         split_users = (ns > 1) if not p["cluster"] else np.zeros_like(ns, dtype=bool)
-    # split users without a cluster go through the merge kernel: it visits one
-    # row per (verify token, query head); (m, l) and D partial outputs per
-    # (split, head, row) in the workspace
-    assert p["n_merge"] == int(((L + 1) * Hq)[split_users].sum())
+    # split users without a cluster go through the merge kernel: (one CTA
+    # per item) it visits one row per (verify token, query head); (m, l) and
+    # D partial outputs per (split, head, row) in the workspace
+    if not p["stream_chunks"]:
+        assert p["n_merge"] == int(((L + 1) * Hq)[split_users].sum())
     part_rows = int((ns * Hkv * G * (L + 1))[split_users].sum())
     assert p["ws_bytes"] >= part_rows * (8 + 4 * D)
     assert (p["ws_bytes"] == 0) == (part_rows == 0)
