@@ -176,12 +176,13 @@ def source_hash(paths):
     return h.hexdigest()[:16]
 
 
-def recorded_traffic(kernel_file, src_hash):
-    """DRAM bytes per launch from the committed ncu summary, if taken on this source."""
+def recorded_traffic(kernel, workload, src_hash):
+    """DRAM bytes (read + write) per launch from the committed ncu summary, if
+    one was taken of this kernel on this workload and this source."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
-            rec = json.load(f).get(kernel_file)
+            rec = json.load(f).get(f"{kernel}@workload{workload}")
     except (OSError, ValueError):
         return None
     if not rec or rec.get("source_hash") != src_hash:
@@ -608,11 +609,11 @@ def write_line(args, b, world, hbm_peak, peak_kind, stages, total_ms_max, units_
     stages["verify_attention_append"]["note"] = ("attention that also writes the verify tokens' K/V rows into "
                                                  "their pages (same launch)")
     # The roofline is the single kernel with the longest launches: the attention
-    # kernel (one launch per stage on this workload), ahead of each of the two
-    # chained spec-verify kernels (see the ncu launch list under profiles/).
+    # kernel (one launch per stage on this workload), ahead of each of the
+    # three chained spec-verify kernels (see the ncu launch list under profiles/).
     dom = "verify_attention"
     ds = stages[dom]
-    traffic = recorded_traffic(dom, source_hash(["paper_2604_20919_gb300/csrc/attention_tc.cuh"]))
+    traffic = recorded_traffic(dom, args.workload, source_hash(["paper_2604_20919_gb300/csrc/attention_tc.cuh"]))
     ms_attn, ms_spec = stages["verify_attention"]["ms"], stages["spec_verify"]["ms"]
     per_step = step_ms / n_steps
     line = {

@@ -219,6 +219,9 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
     const int my_pg = lane < kKBoxes ? kb / kHalves : (vb & (kPages - 1));
     const int my_hf = kb % kHalves;
     int issued = 0;  // tiles issued over all items (the global tile index of the next)
+    // every K/V page is read once per launch (per row block): evict first, so
+    // the stream keeps the split partials and other reused lines in L2
+    const uint64_t kv_pol = l2_evict_first_policy();
     bool alive = true;
     // block ids of page group `group` of the split [kv_begin, kv_end) of the
     // user whose block-table row is `row` (lane = page in the group)
@@ -272,7 +275,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
         }
         if (lane == 0) mbar_arrive_expect_tx(&k_full[st], tp * L::kPageBytes);
         __syncwarp();
-        if (lane < kKBoxes && my_pg < tp) tma_load_4d(sK + koff, &tm_k, my_hf * 64, 0, h, bk, &k_full[st]);
+        if (lane < kKBoxes && my_pg < tp) tma_load_4d_hint(sK + koff, &tm_k, my_hf * 64, 0, h, bk, &k_full[st], kv_pol);
         // V tile
         if (gj >= S && lane == 0) go = mbar_wait(&v_empty[st], ph, p.status);
         if (!__shfl_sync(0xffffffffu, go, 0)) {
@@ -282,7 +285,7 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
         if (lane == 0) mbar_arrive_expect_tx(&v_full[st], tp * L::kPageBytes);
         __syncwarp();
         if (lane >= kKBoxes && lane < kKBoxes + kPages && my_pg < tp)
-          tma_load_5d(sV + voff, &tm_v, 0, 0, 0, h, bk, &v_full[st]);
+          tma_load_5d_hint(sV + voff, &tm_v, 0, 0, 0, h, bk, &v_full[st], kv_pol);
         ++issued;
         if (patched(j)) {
           // the appended rows of this tile, straight from the input, over what
