@@ -621,7 +621,9 @@ verify_attention_tc_kernel(const __grid_constant__ AttnParams<CAP> p, const __gr
       }
       if constexpr (PERSIST) {
         // the first split of a cut stream leaves the stream's merge descriptor
-        if (nsplit > 1 && split == 0 && threadIdx.x == 64) {
+        // (chunk_cut: 255 = no cut stream starts in this chunk; the host
+        // marks exactly the streams this test finds)
+        if (nsplit > 1 && split == 0 && threadIdx.x == 64 && p.chunk_cut[blockIdx.x] != 255) {
           MergeDesc dsc;
           dsc.part_row0 = p.part_off[ui] + static_cast<long long>(h) * M + row0;
           dsc.out_base = static_cast<long long>(U.q_off) * p.Hq + h * p.G;
