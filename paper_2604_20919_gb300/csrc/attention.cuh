@@ -5,9 +5,10 @@
 // This header holds what the attention kernel (attention_tc.cuh) shares with
 // the host: the work parameters (rows r = t*G + g of user i pack its verify
 // tokens and the G query heads of KV head h; a row block is 128 rows), the
-// decoding of a CTA's work, and verify_attention_merge_kernel, which combines
-// the KV splits of one (user, row block, head) through global memory when
-// they do not run as one cluster.
+// decoding of a CTA's work, and the two kernels that combine the KV splits of
+// one (user, row block, head) through global memory when they do not run as
+// one cluster: verify_attention_merge_kernel (one CTA per item plans) and
+// verify_attention_merge_streams_kernel (the streams a persistent grid cut).
 //
 // Two ways to cut the work:
 //   * items (one per CTA): (user, row block, KV head, split), every split of
@@ -19,7 +20,9 @@
 //     streams its chunk covers, in order; the host cuts the chunks so that
 //     every CTA carries about the same pages plus a fixed cost per piece.  A
 //     stream cut by a chunk boundary is merged afterwards, its split s being
-//     its piece in the s-th chunk it touches.
+//     its piece in the s-th chunk it touches.  A CTA finds its first piece
+//     from per-chunk facts the host records and walks to each later one
+//     directly (the next stream), without searching.
 #pragma once
 
 #include "common.cuh"

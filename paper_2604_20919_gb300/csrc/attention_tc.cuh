@@ -22,7 +22,9 @@
 //               released separately: K once its Q K^T has run, V after its
 //               P V.  Page ids are fetched 32 at a time, one per lane, a
 //               group ahead.  A split's last tile loads only the pages up
-//               to the split's end.
+//               to the split's end.  The K/V loads carry an evict-first L2
+//               policy (each page is read once); in a persistent grid the
+//               next two pieces' Q rows are prefetched into L2.
 //   warp 1      allocates TMEM; one thread issues tcgen05.mma as operands
 //               become ready (no fixed order between the two products):
 //                 S[b] = Q K^T      (A = Q from tensor memory, M=128, N=128)
@@ -46,8 +48,10 @@
 // k_patch / v_patch instead of k_full / v_full; the CTA with the last split
 // and the first row block of each (user, head) also writes them into the
 // pages (the round's state update).
-// KV splits: either each split writes (m, l, O) rows to global memory for
-// verify_attention_merge_kernel, or (p.cluster > 1) the splits of one row
+// KV splits: either each split writes (m, l, O) rows to global memory for a
+// merge kernel (in a persistent grid the CTA running a cut stream's first
+// split also writes the stream's merge descriptor), or (p.cluster > 1) the
+// splits of one row
 // block and head run as one thread-block cluster and merge through
 // distributed shared memory: each rank owns a share of the 32-column chunks
 // of O, receives the other ranks' (m, l) rows and their rows of its chunks in
